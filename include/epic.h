@@ -1,0 +1,201 @@
+/*
+ * epic.h -- C-ABI of the GB300 (sm_103a) hot path of EPIC
+ * ("Efficient and Parallel Inference under CFG Constraints for Diffusion
+ * Language Models", arXiv 2606.00722).
+ *
+ * One denoising step of a masked diffusion LM under a context-free grammar:
+ * every (masked position, candidate token) pair is lexed through a memoized
+ * token x lexer-state table and checked for completability by Earley-style
+ * recognition over the partial output's lexeme graph; relaxed compatible
+ * subset selection then picks a parallel commit that is re-checked jointly.
+ *
+ * Conventions (all calls):
+ *   - Every d_* argument is a DEVICE pointer owned by the caller; every other
+ *     pointer is host memory, read during the call only.
+ *   - Token ids are 0..vocab-1; -1 in x means MASK.
+ *   - Batch calls are asynchronous on `cuda_stream` (a cudaStream_t, NULL =
+ *     legacy default stream).  Argument errors are detected on the host and
+ *     returned synchronously before anything is enqueued.  Device-side
+ *     capacity overflow is reported per check (value 2 in d_valid / d_selected)
+ *     and counted in the statistics (epic_get_stats), never silently dropped.
+ *   - The library owns the opaque objects and the device workspace they hold;
+ *     a grammar or lexer table must not be destroyed while work that uses it
+ *     is still in flight.  Calls that share one object must not overlap in
+ *     time on different streams (they share its workspace).
+ *   - There is no CPU fallback: when no CUDA device is usable the calls
+ *     return EPIC_ERR_CUDA.
+ */
+#ifndef EPIC_H_
+#define EPIC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  EPIC_OK = 0,
+  EPIC_ERR_INVALID_ARG = 1, /* bad pointer, size, id, position or NaN          */
+  EPIC_ERR_GRAMMAR = 2,     /* malformed productions, or L(G) is empty          */
+  EPIC_ERR_LEXER = 3,       /* malformed terminal regex, or it matches epsilon  */
+  EPIC_ERR_OOM = 4,         /* host or device allocation failed                 */
+  EPIC_ERR_CUDA = 5,        /* a CUDA call failed (no device, launch error ...) */
+  EPIC_ERR_CAPACITY = 6,    /* a workload exceeded a device capacity limit      */
+  EPIC_ERR_TIMEOUT = 7      /* a bounded device loop ran out of iterations      */
+} epic_status;
+
+typedef struct epic_grammar epic_grammar;         /* grammar + lexer DFA + device tables */
+typedef struct epic_lexer_table epic_lexer_table; /* memoized token x state lex table    */
+
+/*
+ * Grammar description (host memory, copied by epic_grammar_create).
+ * Symbols: terminals are 0..n_terminals-1, nonterminal j is n_terminals+j.
+ * G = (V, Sigma_lex, P, S) of Sec. 3: the terminals are the lexemes.
+ *
+ * terminal_regex[t]: NUL-terminated byte regex.  Syntax: literal bytes;
+ *   `\c` escapes any byte c (`\n`, `\t`, `\r` are newline, tab, CR);
+ *   classes `[a-z_]`, negated `[^"]`, with ranges; `.` = any byte but '\n';
+ *   grouping `( )`; alternation `|`; postfix `*`, `+`, `?`.
+ * terminal_skip[t] = 1 drops the terminal from lexeme sequences (whitespace);
+ *   a skipped terminal may not appear in a production.
+ * Terminal priority is its index: when one lexeme matches several terminals
+ * the lowest index wins.
+ * Productions: lhs[p] in 0..n_nonterminals-1, right-hand side
+ *   rhs[rhs_off[p] .. rhs_off[p+1]-1] (at most 62 symbols; empty = epsilon).
+ */
+typedef struct {
+  int32_t n_terminals;
+  const char* const* terminal_regex;
+  const uint8_t* terminal_skip;
+  int32_t n_nonterminals;
+  int32_t start; /* nonterminal index of S */
+  int32_t n_productions;
+  const int32_t* lhs;
+  const int32_t* rhs_off; /* [n_productions + 1] */
+  const int32_t* rhs;
+} epic_grammar_desc;
+
+/*
+ * Compile a grammar (Alg. 1 line 1-2: compile the lexical map; the regular
+ * cover of Sec. 4.3 / App. A.2 is derived from the same tables).  Builds the
+ * union lexer DFA (minimized), trims unproductive and unreachable symbols,
+ * numbers the dotted items and uploads the device tables to the current
+ * CUDA device.  Errors: EPIC_ERR_INVALID_ARG (NULL / out-of-range ids),
+ * EPIC_ERR_LEXER (bad regex, terminal matching epsilon), EPIC_ERR_GRAMMAR
+ * (empty language), EPIC_ERR_CUDA / EPIC_ERR_OOM.  Synchronous.
+ */
+epic_status epic_grammar_create(const epic_grammar_desc* desc, epic_grammar** out);
+void epic_grammar_destroy(epic_grammar* g);
+
+/* Number of lexer DFA states (the "live lexer states" a span after a gap may
+ * start in, Sec. 2 / Alg. 2), or -1 for NULL. */
+int32_t epic_grammar_lexer_states(const epic_grammar* g);
+
+/*
+ * Build the memoized lexing table (Sec. 4.1, Alg. 2, App. D.1) on the device:
+ * for every token t and lexer state q, the greedy transducer's run of
+ * terminals over t's bytes and its end state (or DEAD).  The rule: at state q
+ * reading byte c, follow delta(q, c) if defined; else, if q accepts, emit its
+ * terminal and restart from delta(q0, c); else DEAD.  Skipped terminals are
+ * not emitted.  Vocabulary (host): token t's bytes are
+ * tok_bytes[tok_off[t] .. tok_off[t+1]-1]; every token has 1..64 bytes.
+ * Table layout in HBM: [vocab][lexer states] entries of 16 bytes.  Enqueued
+ * on cuda_stream; a token whose run exceeds 13 terminals is an
+ * EPIC_ERR_CAPACITY error (checked when the call returns, which synchronizes
+ * the stream once).
+ */
+epic_status epic_lexer_table_build(const epic_grammar* g, const int32_t* tok_off,
+                                   const uint8_t* tok_bytes, int32_t vocab, void* cuda_stream,
+                                   epic_lexer_table** out);
+void epic_lexer_table_destroy(epic_lexer_table* t);
+
+/*
+ * Copy lex-table entries of tokens [first_token, first_token + count) to host
+ * memory (synchronous; for inspection and tests).  Entry (t, q) is 16 bytes:
+ * uint16 end state (0xFFFF = DEAD), uint8 run length, uint8 terminals[13].
+ * host_out must hold count * epic_grammar_lexer_states(g) * 16 bytes.
+ */
+epic_status epic_lexer_table_copy(const epic_lexer_table* t, int32_t first_token, int32_t count,
+                                  void* host_out, size_t out_bytes);
+
+/*
+ * Batched validity checks (Sec. 3; Alg. 3 per check; Alg. 1 line 15):
+ *   d_valid[b][j][c] = Valid_G(x_b, {(d_pos[b][j], d_cand[b][j][c])})
+ *                    = 1[ L(G) cap C_{x_b (+) (pos, tok)} != empty ].
+ * d_x [B][n] int32 (-1 = MASK); d_pos [B][k] int32, each a masked position of
+ * its row; d_cand [B][k][K] int32 token ids; d_valid [B][k][K] uint8 output:
+ * 0 invalid, 1 valid, 2 capacity overflow for that check (no result).
+ * The partial-output graph follows the gap reading of the design notes: each
+ * maximal run of masks is one gap with a Sigma_lex* self-loop, each maximal
+ * run of tokens a span lexed from q0 at the sequence start and from every
+ * lexer state after a gap, flushed at END.  Host-side errors:
+ * EPIC_ERR_INVALID_ARG for sizes < 0 or NULL pointers with non-empty sizes.
+ * Device-side: an unmasked position or an out-of-range token id yields 0 for
+ * that check and counts in stats.bad_inputs.  Asynchronous.
+ */
+epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t,
+                                const int32_t* d_x, int32_t B, int32_t n, const int32_t* d_pos,
+                                int32_t k, const int32_t* d_cand, int32_t K, uint8_t* d_valid,
+                                void* cuda_stream);
+
+/*
+ * Candidate set C of Alg. 1 line 7 under the reading of the design notes:
+ * per proposed position, the highest-confidence candidate whose valid bit is
+ * 1 (ties: lowest candidate index), else none.  d_cand [B][k][K] int32,
+ * d_cand_conf [B][k][K] float32, d_valid [B][k][K] uint8; outputs d_tok [B][k]
+ * int32 (-1 = none) and d_conf [B][k] float32.  Asynchronous.
+ */
+epic_status epic_pick_candidates(const int32_t* d_cand, const float* d_cand_conf,
+                                 const uint8_t* d_valid, int32_t B, int32_t k, int32_t K,
+                                 int32_t* d_tok, float* d_conf, void* cuda_stream);
+
+/*
+ * Relaxed compatible subset selection with exact shrink (Sec. 4.3, Alg. 4),
+ * one sequence per CTA: C = the proposed (position, d_tok) pairs with
+ * d_tok >= 0, sorted by descending d_conf (ties: ascending position);
+ * B = ExactShrink(x, RelaxedSelect(x, C)) where RelaxedSelect's group test is
+ * L(F_G) cap L(A_{x (+) C}) != empty on the flattened regular cover, and
+ * ExactShrink's test is the exact check of the joint update.
+ * d_selected [B][k] uint8: 1 = in the committed batch (|B| >= 2 or none),
+ * 2 = capacity overflow for the sequence (nothing selected).  A NaN
+ * confidence counts as bad input (nothing selected for that sequence).
+ * Asynchronous.
+ */
+epic_status epic_select_compatible_subset(const epic_grammar* g, const epic_lexer_table* t,
+                                          const int32_t* d_x, int32_t B, int32_t n,
+                                          const int32_t* d_pos, int32_t k, const int32_t* d_tok,
+                                          const float* d_conf, uint8_t* d_selected,
+                                          void* cuda_stream);
+
+/*
+ * Commit (Alg. 1 line 10): d_x[b][d_pos[b][j]] = d_tok[b][j] where
+ * d_selected[b][j] == 1.  Asynchronous.
+ */
+epic_status epic_commit(int32_t* d_x, int32_t B, int32_t n, const int32_t* d_pos, int32_t k,
+                        const int32_t* d_tok, const uint8_t* d_selected, void* cuda_stream);
+
+/* Device counters accumulated since the object was created (or reset). */
+typedef struct {
+  uint64_t checks;           /* single-candidate validity checks run           */
+  uint64_t valid;            /* of which valid                                 */
+  uint64_t overflow;         /* checks or selections that hit a capacity limit */
+  uint64_t bad_inputs;       /* unmasked positions / bad token ids / NaNs      */
+  uint64_t columns;          /* Earley chart columns (graph nodes) processed   */
+  uint64_t entries;          /* (node, origin) chart entries stored            */
+  uint64_t cover_checks;     /* regular-cover group tests (Alg. 4 line 9)      */
+  uint64_t exact_checks;     /* joint exact checks (Alg. 4 line 21)            */
+  uint64_t selected;         /* candidates committed by selection              */
+} epic_stats;
+
+/* Copy the counters (synchronizes the lexer table's last stream); out_bytes
+ * must be >= sizeof(epic_stats).  reset != 0 zeroes them afterwards. */
+epic_status epic_get_stats(const epic_lexer_table* t, epic_stats* out, size_t out_bytes, int reset);
+
+const char* epic_status_string(epic_status s);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* EPIC_H_ */

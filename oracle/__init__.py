@@ -111,13 +111,16 @@ class Oracle:
         self._lib.orc_set_vocab(self.h, len(vocab), _p(off, C.c_int32), _p(data, C.c_uint8))
         self.vocab = list(vocab)
 
-    def lex(self, text: bytes, entry: int = 0, flush_end: bool = True):
-        """Greedy lexing of text from live lexer state `entry` (0 = initial).
-        Returns (run of terminal ids, pending state index) or None if DEAD."""
+    def lex(self, text: bytes, entry: int = 0, flush_end: bool = True, run_only: bool = False):
+        """Greedy lexing of text from live lexer state `entry` (0 = initial):
+        with the END flush, or as a span before a gap, or (run_only) with the
+        pending lexeme left open.  Returns (run of terminal ids, pending
+        state index) or None if DEAD."""
         buf = np.frombuffer(text or b'\0', np.uint8).copy()
         out = np.zeros(len(text) + 2, np.int32)
         pend = C.c_int32(-1)
-        r = self._lib.orc_lex(self.h, entry, _p(buf, C.c_uint8), len(text), int(flush_end),
+        mode = 0 if run_only else (1 if flush_end else 2)
+        r = self._lib.orc_lex(self.h, entry, _p(buf, C.c_uint8), len(text), mode,
                               _p(out, C.c_int32), len(out), C.byref(pend))
         if r == -1:
             return None

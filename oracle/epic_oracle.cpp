@@ -240,8 +240,19 @@ bool extensible(const Grammar& g, const std::vector<int>& q) {
 // some byte could extend it (the gap absorbs its terminal); a lexeme that no
 // byte can extend has ended, so an accepting state emits its terminal.
 // Skipped terminals are dropped from the run.  Returns false on DEAD.
+enum LexEnd { kRunOnly = 0, kEndFlush = 1, kBeforeGap = 2 };
+
+bool lex_run_mode(const Grammar& g, const std::vector<int>& entry, const std::string& bytes, int mode,
+                  std::vector<int>& run, std::vector<int>& pending);
+
 bool lex_run(const Grammar& g, const std::vector<int>& entry, const std::string& bytes,
              bool flush_end, std::vector<int>& run, std::vector<int>& pending) {
+  return lex_run_mode(g, entry, bytes, flush_end ? kEndFlush : kBeforeGap, run, pending);
+}
+
+bool lex_run_mode(const Grammar& g, const std::vector<int>& entry, const std::string& bytes, int mode,
+                  std::vector<int>& run, std::vector<int>& pending) {
+  bool flush_end = mode == kEndFlush;
   std::vector<int> q = entry;
   run.clear();
   for (unsigned char c : bytes) {
@@ -256,7 +267,7 @@ bool lex_run(const Grammar& g, const std::vector<int>& entry, const std::string&
     q = step(g, g.q0, c);
     if (q.empty()) return false;
   }
-  if (!flush_end && q != g.q0 && !extensible(g, q)) {
+  if (mode == kBeforeGap && q != g.q0 && !extensible(g, q)) {
     int t = accepts(g, q);
     if (t < 0) return false;
     if (!g.skip[t]) run.push_back(t);
@@ -759,13 +770,14 @@ void orc_set_vocab(void* h, int V, const int* off, const uint8_t* bytes) {
 }
 
 // Lex a byte string from lexer state `entry` (index into the live states,
-// 0 = q0).  Returns the run length, -1 if DEAD, -2 if cap is too small.
-// *pending receives the index of the pending state.
-int orc_lex(void* h, int entry, const uint8_t* s, int len, int flush_end, int* out, int cap,
+// 0 = q0).  mode: 0 = the run only (pending lexeme left open), 1 = END
+// flush, 2 = a gap follows.  Returns the run length, -1 if DEAD, -2 if cap
+// is too small.  *pending receives the index of the pending state.
+int orc_lex(void* h, int entry, const uint8_t* s, int len, int mode, int* out, int cap,
             int* pending) {
   Grammar& g = ((Oracle*)h)->g;
   std::vector<int> run, pend;
-  if (!lex_run(g, g.states[entry], std::string((const char*)s, len), flush_end != 0, run, pend))
+  if (!lex_run_mode(g, g.states[entry], std::string((const char*)s, len), mode, run, pend))
     return -1;
   if ((int)run.size() > cap) return -2;
   std::copy(run.begin(), run.end(), out);

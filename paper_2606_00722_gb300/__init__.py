@@ -1,0 +1,5 @@
+"""GB300 (sm_103a) hot path of EPIC (arXiv 2606.00722): batched validity
+checking of candidate commits under a CFG, relaxed compatible subset
+selection and commit, behind the C-ABI of ``include/epic.h``."""
+from .epic import (Grammar, LexTable, EpicError, build, load, validate_batch,  # noqa: F401
+                   pick_candidates, select_compatible_subset, commit, LIB_PATH, EXPORTS)

@@ -1,0 +1,778 @@
+// Kernels and C-ABI of the EPIC hot path on sm_103a (see include/epic.h).
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstring>
+#include <new>
+#include <stdexcept>
+#include <string>
+#include <vector>
+
+#include "../../include/epic.h"
+#include "grammar.h"
+#include "skeleton.cuh"
+
+using namespace epic;
+
+// ================================================================ kernels
+
+// K1: memoized lex table.  One thread per (token, entry state); consecutive
+// threads share a token (its bytes are a broadcast read) and write
+// consecutive 16-byte entries.
+__global__ void k_lex_table(const int32_t* __restrict__ tok_off, const uint8_t* __restrict__ bytes, int vocab,
+                            int Q, const int32_t* __restrict__ dfa_next, const int16_t* __restrict__ dfa_acc,
+                            const uint8_t* __restrict__ skip, LexEntry* __restrict__ table, int* overflow) {
+  long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (long long)vocab * Q) return;
+  int t = (int)(idx / Q), q = (int)(idx % Q);
+  LexEntry e;
+  uint32_t* raw = reinterpret_cast<uint32_t*>(&e);
+  raw[0] = raw[1] = raw[2] = raw[3] = 0;
+  int s = q, len = 0;
+  bool dead = false;
+  for (int i = tok_off[t]; i < tok_off[t + 1]; ++i) {
+    int c = bytes[i];
+    int nx = dfa_next[s * 256 + c];
+    if (nx >= 0) {
+      s = nx;
+      continue;
+    }
+    int a = dfa_acc[s];  // q0 never accepts (no terminal matches epsilon)
+    if (a < 0) {
+      dead = true;
+      break;
+    }
+    if (!skip[a]) {
+      if (len >= 13) {
+        atomicExch(overflow, 1);
+        dead = true;
+        break;
+      }
+      e.term[len++] = (uint8_t)a;
+    }
+    s = dfa_next[c];  // restart from q0 on c
+    if (s < 0) {
+      dead = true;
+      break;
+    }
+  }
+  e.end = dead ? 0xFFFF : (uint16_t)s;
+  e.len = dead ? 0 : (uint8_t)len;
+  table[idx] = e;
+}
+
+struct WsPack {
+  char* base;
+  size_t per_cta;
+  WsDims dims;
+  int W, VW, FW;
+  __device__ void carve(int cta, Workspace& ws, WalkScratch& sc) const {
+    char* p = base + per_cta * (size_t)cta;
+    auto take = [&](size_t bytes) {
+      char* r = p;
+      p += (bytes + 255) & ~(size_t)255;
+      return r;
+    };
+    int nm = dims.nmax;
+    ws.stage = (uint32_t*)take((size_t)nm * W * 4);
+    ws.bdone = (uint32_t*)take((size_t)nm * VW * 4);
+    ws.col_off = (int32_t*)take((size_t)(nm + 1) * 4);
+    ws.cov = (uint32_t*)take((size_t)nm * FW * 4);
+    sc.g_src = (int32_t*)take(kMaxQ * 4);
+    sc.g_end = (int32_t*)take(kMaxQ * 4);
+    sc.g_len = (int32_t*)take(kMaxQ * 4);
+    sc.g_last = (int32_t*)take(kMaxQ * 4);
+    sc.f_q = (int32_t*)take(kMaxQ * 4);
+    sc.f_c = (int32_t*)take(kMaxQ * 4);
+    sc.key_q = (int32_t*)take(kMaxQ * 4);
+    sc.g_tail = (uint8_t*)take(kMaxQ * 16);
+    sc.g_lbl = (uint32_t*)take(kMaxQ * 8 * 4);
+    sc.expn = (uint32_t*)take((size_t)nm * W * 4);
+    sc.bnew = (uint32_t*)take((size_t)nm * VW * 4);
+    ws.org = (int32_t*)take((size_t)dims.emax * 4);
+    ws.bits = (uint32_t*)take((size_t)dims.emax * W * 4);
+  }
+};
+
+static size_t ws_bytes_per_cta(const WsDims& d, int W, int VW, int FW) {
+  auto r = [](size_t b) { return (b + 255) & ~(size_t)255; };
+  size_t nm = d.nmax;
+  return r(nm * W * 4) + r(nm * VW * 4) + r((nm + 1) * 4) + r(nm * FW * 4) + 7 * r(kMaxQ * 4) +
+         r(kMaxQ * 16) + r(kMaxQ * 32) + r(nm * W * 4) + r(nm * VW * 4) + r((size_t)d.emax * 4) +
+         r((size_t)d.emax * W * 4);
+}
+
+enum StatIdx { S_CHECKS, S_VALID, S_OVERFLOW, S_BAD, S_COLUMNS, S_ENTRIES, S_COVER, S_EXACT, S_SELECTED, S_N };
+
+// K2-K4: one CTA per validity check (persistent CTAs pull checks from a
+// counter).  Each check walks the lexeme graph of x (+) (pos, tok) and runs
+// bit-parallel Earley recognition over it.
+__global__ void __launch_bounds__(kThreads) k_validate(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
+                                                       const int32_t* __restrict__ x, int n, const int32_t* __restrict__ pos,
+                                                       int k, const int32_t* __restrict__ cand, int K, long long total,
+                                                       uint8_t* __restrict__ valid, WsPack wsp,
+                                                       unsigned long long* counter, unsigned long long* stats) {
+  __shared__ WalkShared sh;
+  __shared__ long long job;
+  Workspace ws;
+  WalkScratch sc;
+  wsp.carve(blockIdx.x, ws, sc);
+  EarleyCols cols(g, table, ws, sc, wsp.dims, sh);
+  Walk<EarleyCols> walk(cols, g, table, sc, sh, vocab);
+  for (;;) {
+    if (threadIdx.x == 0) job = (long long)atomicAdd(counter, 1ull);
+    __syncthreads();
+    long long jb = job;
+    if (jb >= total) break;
+    long long b = jb / ((long long)k * K);
+    long long j = (jb / K) % k;
+    Subst s{pos + b * k + j, cand + jb, 1};
+    int r = walk.run(x + b * n, n, s);
+    if (threadIdx.x == 0) {
+      valid[jb] = r == 1 ? 1 : (r == -1 ? 2 : 0);
+      atomicAdd(&stats[S_CHECKS], 1ull);
+      if (r == 1) atomicAdd(&stats[S_VALID], 1ull);
+      if (r == -1) atomicAdd(&stats[S_OVERFLOW], 1ull);
+      if (r == -2) atomicAdd(&stats[S_BAD], 1ull);
+      atomicAdd(&stats[S_COLUMNS], (unsigned long long)sh.ncols);
+      atomicAdd(&stats[S_ENTRIES], (unsigned long long)sh.nent);
+    }
+    __syncthreads();
+  }
+}
+
+// Per proposed position: the highest-confidence candidate with valid bit 1.
+__global__ void k_pick(const int32_t* __restrict__ cand, const float* __restrict__ conf,
+                       const uint8_t* __restrict__ valid, int B, int k, int K, int32_t* __restrict__ tok,
+                       float* __restrict__ out_conf) {
+  long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (long long)B * k) return;
+  int best = -1;
+  float bc = 0.f;
+  for (int c = 0; c < K; ++c) {
+    long long q = i * K + c;
+    if (valid[q] != 1) continue;
+    float v = conf[q];
+    if (best < 0 || v > bc) {
+      best = c;
+      bc = v;
+    }
+  }
+  tok[i] = best < 0 ? -1 : cand[i * K + best];
+  out_conf[i] = best < 0 ? 0.f : bc;
+}
+
+// Alg. 4 per sequence: one CTA runs RelaxedSelect / ExactShrink with an
+// explicit stack; thread 0 drives the recursion, the whole CTA runs each
+// cover test (CoverCols walk) and exact joint check (EarleyCols walk).
+constexpr int kMaxSel = 64;
+
+struct SelFrame {
+  int8_t kind;  // 0 root, 1 relaxed, 2 shrink
+  int8_t pc;
+  unsigned long long base, set, a, b;
+};
+
+__global__ void __launch_bounds__(kThreads) k_select(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
+                                                     const int32_t* __restrict__ x, int B, int n,
+                                                     const int32_t* __restrict__ pos, int k,
+                                                     const int32_t* __restrict__ tok, const float* __restrict__ conf,
+                                                     uint8_t* __restrict__ selected, WsPack wsp,
+                                                     unsigned long long* stats) {
+  __shared__ WalkShared sh;
+  __shared__ int c_slot[kMaxSel], c_pos[kMaxSel], c_tok[kMaxSel];
+  __shared__ int s_pos[kMaxSel], s_tok[kMaxSel];
+  __shared__ SelFrame stack[2 * kMaxSel + 8];
+  __shared__ int sp, nc, action, result, bad, overflow;
+  __shared__ unsigned long long ret, final_set;
+  Workspace ws;
+  WalkScratch sc;
+  wsp.carve(blockIdx.x, ws, sc);
+  EarleyCols ecols(g, table, ws, sc, wsp.dims, sh);
+  CoverCols ccols(g, ws, wsp.dims, sh);
+  Walk<EarleyCols> exact(ecols, g, table, sc, sh, vocab);
+  Walk<CoverCols> cover(ccols, g, table, sc, sh, vocab);
+  for (int b = blockIdx.x; b < B; b += gridDim.x) {
+    const int32_t* xb = x + (long long)b * n;
+    if (threadIdx.x == 0) {
+      // C: proposed (position, token) pairs, by descending confidence then
+      // ascending position (insertion sort; k <= 64)
+      int m = 0;
+      bad = 0;
+      overflow = 0;
+      for (int j = 0; j < k; ++j) {
+        int t = tok[(long long)b * k + j];
+        if (t < 0) continue;
+        float cf = conf[(long long)b * k + j];
+        if (cf != cf) bad = 1;
+        int p = pos[(long long)b * k + j];
+        int i = m++;
+        while (i > 0) {
+          float cp = conf[(long long)b * k + c_slot[i - 1]];
+          if (cp > cf || (cp == cf && c_pos[i - 1] < p)) break;
+          c_slot[i] = c_slot[i - 1];
+          c_pos[i] = c_pos[i - 1];
+          c_tok[i] = c_tok[i - 1];
+          --i;
+        }
+        c_slot[i] = j;
+        c_pos[i] = p;
+        c_tok[i] = t;
+      }
+      nc = m;
+      sp = 0;
+      stack[0] = SelFrame{0, 0, 0ull, nc == 64 ? ~0ull : ((1ull << nc) - 1), 0ull, 0ull};
+      sp = 1;
+      final_set = 0;
+      if (bad) sp = 0;
+    }
+    __syncthreads();
+    for (;;) {
+      // thread 0 advances the recursion until it needs a test or finishes
+      if (threadIdx.x == 0) {
+        action = 0;
+        while (sp > 0 && action == 0) {
+          if (sp >= 2 * kMaxSel + 6) {  // recursion deeper than Alg. 4 can go
+            overflow = 1;
+            sp = 0;
+            break;
+          }
+          SelFrame& f = stack[sp - 1];
+          unsigned long long set = f.set;
+          // split in confidence order: first ceil(|set|/2) members
+          auto halves = [&](unsigned long long s, unsigned long long& L, unsigned long long& R) {
+            int cnt = __popcll(s), h = (cnt + 1) / 2;
+            L = 0;
+            unsigned long long r = s;
+            for (int i = 0; i < h; ++i) {
+              unsigned long long lo = r & (~r + 1);
+              L |= lo;
+              r &= r - 1;
+            }
+            R = s & ~L;
+          };
+          if (f.kind == 0) {
+            if (f.pc == 0) {
+              f.pc = 1;
+              stack[sp++] = SelFrame{1, 0, 0ull, set, 0ull, 0ull};
+            } else if (f.pc == 1) {
+              f.pc = 2;
+              stack[sp++] = SelFrame{2, 0, 0ull, ret, 0ull, 0ull};
+            } else {
+              final_set = ret;
+              --sp;
+            }
+          } else if (f.kind == 1) {  // RelaxedSelect(x (+) base, set)
+            if (f.pc == 0) {
+              if (__popcll(set) <= 1) {
+                ret = 0;
+                --sp;
+              } else {
+                f.pc = 1;
+                action = 1;  // cover test of base | set
+                f.a = f.base | set;
+              }
+            } else if (f.pc == 1) {
+              if (result == 1) {
+                ret = set;
+                --sp;
+              } else {
+                unsigned long long L, R;
+                halves(set, L, R);
+                f.a = R;
+                f.pc = 2;
+                stack[sp++] = SelFrame{1, 0, f.base, L, 0ull, 0ull};
+              }
+            } else if (f.pc == 2) {
+              f.b = ret;
+              f.pc = 3;
+              unsigned long long R = f.a;
+              stack[sp++] = SelFrame{1, 0, f.base | ret, R, 0ull, 0ull};
+            } else {
+              ret = f.b | ret;
+              --sp;
+            }
+          } else {  // ExactShrink(x (+) base, set)
+            if (f.pc == 0) {
+              if (__popcll(set) <= 1) {
+                ret = 0;
+                --sp;
+              } else {
+                f.pc = 1;
+                action = 2;  // exact joint check of base | set
+                f.a = f.base | set;
+              }
+            } else if (f.pc == 1) {
+              if (result == 1) {
+                ret = set;
+                --sp;
+              } else {
+                unsigned long long L, R;
+                halves(set, L, R);
+                f.a = R;
+                f.pc = 2;
+                stack[sp++] = SelFrame{2, 0, f.base, L, 0ull, 0ull};
+              }
+            } else if (f.pc == 2) {
+              f.b = ret;  // B'_L
+              f.pc = 3;
+              stack[sp++] = SelFrame{1, 0, f.base | ret, f.a, 0ull, 0ull};
+            } else if (f.pc == 3) {
+              f.pc = 4;
+              stack[sp++] = SelFrame{2, 0, f.base | f.b, ret, 0ull, 0ull};
+            } else {
+              ret = f.b | ret;
+              --sp;
+            }
+          }
+        }
+        if (action != 0) {
+          unsigned long long m = stack[sp - 1].a;
+          int ns = 0;
+          for (int i = 0; i < nc; ++i)
+            if ((m >> i) & 1ull) {
+              s_pos[ns] = c_pos[i];
+              s_tok[ns] = c_tok[i];
+              ++ns;
+            }
+          result = ns;  // substitution count for the test
+        }
+      }
+      __syncthreads();
+      int act = action;
+      if (act == 0) break;
+      Subst s{s_pos, s_tok, result};
+      __syncthreads();
+      int r = (act == 1) ? cover.run(xb, n, s) : exact.run(xb, n, s);
+      if (threadIdx.x == 0) {
+        if (r < 0) {
+          overflow |= (r == -1);
+          bad |= (r == -2);
+          sp = 0;
+        }
+        result = r == 1 ? 1 : 0;
+        atomicAdd(&stats[act == 1 ? S_COVER : S_EXACT], 1ull);
+      }
+      __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+      for (int j = 0; j < k; ++j) selected[(long long)b * k + j] = overflow ? 2 : 0;
+      if (!overflow && !bad) {
+        for (int i = 0; i < nc; ++i)
+          if ((final_set >> i) & 1ull) selected[(long long)b * k + c_slot[i]] = 1;
+        atomicAdd(&stats[S_SELECTED], (unsigned long long)__popcll(final_set));
+      }
+      if (bad) atomicAdd(&stats[S_BAD], 1ull);
+      if (overflow) atomicAdd(&stats[S_OVERFLOW], 1ull);
+    }
+    __syncthreads();
+  }
+}
+
+__global__ void k_commit(int32_t* __restrict__ x, int B, int n, const int32_t* __restrict__ pos, int k,
+                         const int32_t* __restrict__ tok, const uint8_t* __restrict__ sel) {
+  long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (long long)B * k) return;
+  if (sel[i] != 1) return;
+  long long b = i / k;
+  int p = pos[i];
+  if (p >= 0 && p < n) x[b * n + p] = tok[i];
+}
+
+// ================================================================ host side
+
+struct epic_grammar {
+  int device = 0;
+  GrammarTables tabs;
+  LexerDFA dfa;
+  CoverTables cov;
+  DevGrammar dg{};
+  std::vector<void*> dev_allocs;
+};
+
+struct epic_lexer_table {
+  const epic_grammar* g = nullptr;
+  int vocab = 0;
+  LexEntry* d_table = nullptr;
+  char* d_ws = nullptr;
+  size_t ws_bytes = 0;
+  WsDims dims{};
+  int ctas = 0;
+  unsigned long long* d_stats = nullptr;
+  unsigned long long* d_counter = nullptr;
+  cudaStream_t last = nullptr;
+};
+
+namespace {
+
+template <class T>
+epic_status upload(epic_grammar* g, const std::vector<T>& v, const T** out) {
+  void* p = nullptr;
+  size_t bytes = std::max<size_t>(sizeof(T), v.size() * sizeof(T));
+  if (cudaMalloc(&p, bytes) != cudaSuccess) return EPIC_ERR_OOM;
+  g->dev_allocs.push_back(p);
+  if (!v.empty() && cudaMemcpy(p, v.data(), v.size() * sizeof(T), cudaMemcpyHostToDevice) != cudaSuccess)
+    return EPIC_ERR_CUDA;
+  *out = (const T*)p;
+  return EPIC_OK;
+}
+
+int sm_count() {
+  int dev = 0, n = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  return n > 0 ? n : 1;
+}
+
+// Workspace sizing: columns <= 4096 per walk, entries as many as the budget
+// allows for the CTA count.  EPIC_WORKSPACE_MB (default 8192) caps the total.
+epic_status ensure_workspace(epic_lexer_table* t, int want_ctas, cudaStream_t st) {
+  const epic_grammar* g = t->g;
+  size_t budget_mb = 8192;
+  if (const char* e = getenv("EPIC_WORKSPACE_MB")) budget_mb = strtoull(e, nullptr, 10);
+  int W = g->dg.W, VW = g->dg.VW, FW = g->dg.FW;
+  WsDims d;
+  d.nmax = kMaxCols;
+  long long emax_cap = 1ll << 22;
+  if (const char* e = getenv("EPIC_ENTRIES_PER_CTA")) emax_cap = atoll(e);
+  int ctas = std::max(1, want_ctas);
+  size_t budget = budget_mb << 20;
+  for (;;) {
+    WsDims probe = d;
+    probe.emax = 0;
+    size_t fixed = ws_bytes_per_cta(probe, W, VW, FW);
+    long long per_entry = (long long)(W + 1) * 4;
+    long long room = (long long)(budget / ctas) - (long long)fixed;
+    d.emax = std::min<long long>(emax_cap, room / per_entry);
+    if (d.emax >= 4096 || ctas == 1) break;
+    ctas = std::max(1, ctas / 2);
+  }
+  if (d.emax < 64) return EPIC_ERR_OOM;
+  size_t per = ws_bytes_per_cta(d, W, VW, FW);
+  size_t need = per * (size_t)ctas;
+  if (t->d_ws && t->ws_bytes >= need && t->dims.nmax == d.nmax && t->dims.emax == d.emax) {
+    t->ctas = ctas;
+    return EPIC_OK;
+  }
+  if (t->d_ws) {
+    cudaStreamSynchronize(t->last);
+    cudaFree(t->d_ws);
+    t->d_ws = nullptr;
+  }
+  if (cudaMalloc(&t->d_ws, need) != cudaSuccess) {
+    t->d_ws = nullptr;
+    return EPIC_ERR_OOM;
+  }
+  // staging rows and bdone must start at zero; the rest is written before read
+  if (cudaMemsetAsync(t->d_ws, 0, need, st) != cudaSuccess) return EPIC_ERR_CUDA;
+  t->ws_bytes = need;
+  t->dims = d;
+  t->ctas = ctas;
+  return EPIC_OK;
+}
+
+WsPack pack_of(const epic_lexer_table* t) {
+  WsPack p;
+  p.base = t->d_ws;
+  p.dims = t->dims;
+  p.W = t->g->dg.W;
+  p.VW = t->g->dg.VW;
+  p.FW = t->g->dg.FW;
+  p.per_cta = ws_bytes_per_cta(t->dims, p.W, p.VW, p.FW);
+  return p;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* epic_status_string(epic_status s) {
+  switch (s) {
+    case EPIC_OK: return "ok";
+    case EPIC_ERR_INVALID_ARG: return "invalid argument";
+    case EPIC_ERR_GRAMMAR: return "invalid grammar (malformed or empty language)";
+    case EPIC_ERR_LEXER: return "invalid lexer specification";
+    case EPIC_ERR_OOM: return "out of memory";
+    case EPIC_ERR_CUDA: return "CUDA error";
+    case EPIC_ERR_CAPACITY: return "capacity exceeded";
+    case EPIC_ERR_TIMEOUT: return "device loop bound exceeded";
+  }
+  return "unknown status";
+}
+
+epic_status epic_grammar_create(const epic_grammar_desc* desc, epic_grammar** out) {
+  if (!desc || !out) return EPIC_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (desc->n_terminals <= 0 || desc->n_terminals > 255 || desc->n_nonterminals <= 0 ||
+      desc->n_nonterminals > 32 * kMaxVW || desc->n_productions < 0 || !desc->terminal_regex ||
+      !desc->terminal_skip || (desc->n_productions > 0 && (!desc->lhs || !desc->rhs_off)))
+    return EPIC_ERR_INVALID_ARG;
+  int dev_count = 0;
+  if (cudaGetDeviceCount(&dev_count) != cudaSuccess || dev_count == 0) return EPIC_ERR_CUDA;
+  epic_grammar* g = new (std::nothrow) epic_grammar();
+  if (!g) return EPIC_ERR_OOM;
+  cudaGetDevice(&g->device);
+  int T = desc->n_terminals, V = desc->n_nonterminals, P = desc->n_productions;
+  try {
+    std::vector<std::string> rx;
+    for (int t = 0; t < T; ++t) {
+      if (!desc->terminal_regex[t]) throw std::invalid_argument("null regex");
+      rx.emplace_back(desc->terminal_regex[t]);
+    }
+    try {
+      g->dfa = build_lexer(rx);
+    } catch (std::runtime_error&) {
+      delete g;
+      return EPIC_ERR_LEXER;
+    }
+    if (g->dfa.Q > kMaxQ) {
+      delete g;
+      return EPIC_ERR_CAPACITY;
+    }
+    std::vector<uint8_t> skip(desc->terminal_skip, desc->terminal_skip + T);
+    std::vector<int32_t> lhs(desc->lhs, desc->lhs + P);
+    std::vector<int32_t> off(desc->rhs_off, desc->rhs_off + P + 1);
+    if (off[0] != 0) throw std::invalid_argument("rhs_off[0] != 0");
+    std::vector<int32_t> rhs;
+    if (off[P] > 0) {
+      if (!desc->rhs) throw std::invalid_argument("null rhs");
+      rhs.assign(desc->rhs, desc->rhs + off[P]);
+    }
+    try {
+      g->tabs = build_tables(T, skip, V, desc->start, lhs, off, rhs);
+    } catch (std::domain_error&) {
+      delete g;
+      return EPIC_ERR_GRAMMAR;
+    }
+  } catch (std::exception&) {
+    delete g;
+    return EPIC_ERR_INVALID_ARG;
+  }
+  GrammarTables& G = g->tabs;
+  if (G.W > kMaxW) {
+    delete g;
+    return EPIC_ERR_CAPACITY;
+  }
+  g->cov = build_cover(G);
+  if (g->cov.FW > kMaxFW) {
+    delete g;
+    return EPIC_ERR_CAPACITY;
+  }
+  DevGrammar& d = g->dg;
+  d.T = G.T;
+  d.V = G.V;
+  d.D = G.D;
+  d.W = G.W;
+  d.VW = (G.V + 31) / 32;
+  d.Q = g->dfa.Q;
+  d.start_item = G.start_item;
+  d.accept_item = G.accept_item;
+  std::vector<uint32_t> next_any(G.W);
+  for (int w = 0; w < G.W; ++w) next_any[w] = G.any_term[w] | G.any_nt[w];
+  std::vector<int16_t> inext(G.D), ilhs(G.D);
+  for (int i = 0; i < G.D; ++i) {
+    inext[i] = (int16_t)G.item_next[i];
+    ilhs[i] = (int16_t)G.item_lhs[i];
+  }
+  epic_status st = EPIC_OK;
+  auto up = [&](auto& v, auto** o) {
+    if (st == EPIC_OK) st = upload(g, v, o);
+  };
+  up(G.exp_term, &d.exp_term);
+  up(G.exp_nt, &d.exp_nt);
+  up(G.any_nt, &d.any_nt);
+  up(next_any, &d.next_any);
+  up(G.nullable_next, &d.nullable_next);
+  up(G.complete, &d.complete);
+  up(G.pred, &d.pred);
+  up(G.gap_pred, &d.gap_pred);
+  up(inext, &d.item_next);
+  up(ilhs, &d.item_lhs);
+  up(g->dfa.accept, &d.dfa_accept);
+  up(g->dfa.next, &d.dfa_next);
+  std::vector<uint8_t> ext(g->dfa.Q, 0);
+  for (int q = 0; q < g->dfa.Q; ++q)
+    for (int c = 0; c < 256; ++c)
+      if (g->dfa.next[(size_t)q * 256 + c] >= 0) ext[q] = 1;
+  up(ext, &d.dfa_ext);
+  up(G.skip, &d.skip);
+  d.FS = g->cov.FS;
+  d.FW = g->cov.FW;
+  d.cov_start = g->cov.start;
+  d.cov_accept = g->cov.accept;
+  up(g->cov.eps_close, &d.cov_eps_close);
+  up(g->cov.all_close, &d.cov_all_close);
+  if (st != EPIC_OK) {
+    epic_grammar_destroy(g);
+    return st;
+  }
+  *out = g;
+  return EPIC_OK;
+}
+
+void epic_grammar_destroy(epic_grammar* g) {
+  if (!g) return;
+  for (void* p : g->dev_allocs) cudaFree(p);
+  delete g;
+}
+
+int32_t epic_grammar_lexer_states(const epic_grammar* g) { return g ? g->dfa.Q : -1; }
+
+epic_status epic_lexer_table_build(const epic_grammar* g, const int32_t* tok_off, const uint8_t* tok_bytes,
+                                   int32_t vocab, void* cuda_stream, epic_lexer_table** out) {
+  if (!g || !tok_off || !out || vocab <= 0) return EPIC_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (tok_off[0] != 0) return EPIC_ERR_INVALID_ARG;
+  for (int t = 0; t < vocab; ++t) {
+    int L = tok_off[t + 1] - tok_off[t];
+    if (L < 1 || L > 64) return EPIC_ERR_INVALID_ARG;
+  }
+  if (!tok_bytes) return EPIC_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  epic_lexer_table* t = new (std::nothrow) epic_lexer_table();
+  if (!t) return EPIC_ERR_OOM;
+  t->g = g;
+  t->vocab = vocab;
+  t->last = st;
+  int Q = g->dg.Q;
+  size_t nbytes = (size_t)tok_off[vocab];
+  int32_t* d_off = nullptr;
+  uint8_t* d_bytes = nullptr;
+  int* d_ovf = nullptr;
+  epic_status res = EPIC_OK;
+  if (cudaMalloc(&t->d_table, (size_t)vocab * Q * sizeof(LexEntry)) != cudaSuccess ||
+      cudaMalloc(&d_off, (size_t)(vocab + 1) * 4) != cudaSuccess || cudaMalloc(&d_bytes, nbytes) != cudaSuccess ||
+      cudaMalloc(&d_ovf, 4) != cudaSuccess || cudaMalloc(&t->d_stats, S_N * 8) != cudaSuccess ||
+      cudaMalloc(&t->d_counter, 8) != cudaSuccess) {
+    res = EPIC_ERR_OOM;
+  }
+  if (res == EPIC_OK) {
+    cudaMemcpyAsync(d_off, tok_off, (size_t)(vocab + 1) * 4, cudaMemcpyHostToDevice, st);
+    cudaMemcpyAsync(d_bytes, tok_bytes, nbytes, cudaMemcpyHostToDevice, st);
+    cudaMemsetAsync(d_ovf, 0, 4, st);
+    cudaMemsetAsync(t->d_stats, 0, S_N * 8, st);
+    long long total = (long long)vocab * Q;
+    int threads = 256;
+    long long blocks = (total + threads - 1) / threads;
+    k_lex_table<<<(unsigned)blocks, threads, 0, st>>>(d_off, d_bytes, vocab, Q, g->dg.dfa_next, g->dg.dfa_accept,
+                                                       g->dg.skip, t->d_table, d_ovf);
+    int ovf = 0;
+    if (cudaGetLastError() != cudaSuccess || cudaMemcpyAsync(&ovf, d_ovf, 4, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess)
+      res = EPIC_ERR_CUDA;
+    else if (ovf)
+      res = EPIC_ERR_CAPACITY;
+  }
+  cudaFree(d_off);
+  cudaFree(d_bytes);
+  cudaFree(d_ovf);
+  if (res != EPIC_OK) {
+    epic_lexer_table_destroy(t);
+    return res;
+  }
+  *out = t;
+  return EPIC_OK;
+}
+
+void epic_lexer_table_destroy(epic_lexer_table* t) {
+  if (!t) return;
+  if (t->last) cudaStreamSynchronize(t->last);
+  cudaFree(t->d_table);
+  cudaFree(t->d_ws);
+  cudaFree(t->d_stats);
+  cudaFree(t->d_counter);
+  delete t;
+}
+
+epic_status epic_lexer_table_copy(const epic_lexer_table* t, int32_t first_token, int32_t count, void* host_out,
+                                  size_t out_bytes) {
+  if (!t || !host_out || first_token < 0 || count < 0 || first_token + count > t->vocab) return EPIC_ERR_INVALID_ARG;
+  size_t Q = (size_t)t->g->dg.Q;
+  size_t bytes = (size_t)count * Q * sizeof(LexEntry);
+  if (out_bytes < bytes) return EPIC_ERR_INVALID_ARG;
+  if (cudaStreamSynchronize(t->last) != cudaSuccess) return EPIC_ERR_CUDA;
+  if (cudaMemcpy(host_out, t->d_table + (size_t)first_token * Q, bytes, cudaMemcpyDeviceToHost) != cudaSuccess)
+    return EPIC_ERR_CUDA;
+  return EPIC_OK;
+}
+
+epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* tc, const int32_t* d_x, int32_t B,
+                                int32_t n, const int32_t* d_pos, int32_t k, const int32_t* d_cand, int32_t K,
+                                uint8_t* d_valid, void* cuda_stream) {
+  epic_lexer_table* t = const_cast<epic_lexer_table*>(tc);
+  if (!g || !t || t->g != g || B < 0 || n < 0 || k < 0 || K < 0) return EPIC_ERR_INVALID_ARG;
+  long long total = (long long)B * k * K;
+  if (total == 0) return EPIC_OK;
+  if (!d_x || !d_pos || !d_cand || !d_valid || n == 0) return EPIC_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  int want = (int)std::min<long long>(total, (long long)sm_count() * 2);
+  epic_status s = ensure_workspace(t, want, st);
+  if (s != EPIC_OK) return s;
+  t->last = st;
+  cudaMemsetAsync(t->d_counter, 0, 8, st);
+  k_validate<<<t->ctas, kThreads, 0, st>>>(g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total, d_valid,
+                                           pack_of(t), t->d_counter, t->d_stats);
+  return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
+}
+
+epic_status epic_pick_candidates(const int32_t* d_cand, const float* d_cand_conf, const uint8_t* d_valid, int32_t B,
+                                 int32_t k, int32_t K, int32_t* d_tok, float* d_conf, void* cuda_stream) {
+  if (B < 0 || k < 0 || K < 0) return EPIC_ERR_INVALID_ARG;
+  long long total = (long long)B * k;
+  if (total == 0) return EPIC_OK;
+  if (!d_cand || !d_cand_conf || !d_valid || !d_tok || !d_conf) return EPIC_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  k_pick<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(d_cand, d_cand_conf, d_valid, B, k, K, d_tok, d_conf);
+  return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
+}
+
+epic_status epic_select_compatible_subset(const epic_grammar* g, const epic_lexer_table* tc, const int32_t* d_x,
+                                          int32_t B, int32_t n, const int32_t* d_pos, int32_t k,
+                                          const int32_t* d_tok, const float* d_conf, uint8_t* d_selected,
+                                          void* cuda_stream) {
+  epic_lexer_table* t = const_cast<epic_lexer_table*>(tc);
+  if (!g || !t || t->g != g || B < 0 || n < 0 || k < 0 || k > kMaxSel) return EPIC_ERR_INVALID_ARG;
+  if ((long long)B * k == 0) return EPIC_OK;
+  if (!d_x || !d_pos || !d_tok || !d_conf || !d_selected || n == 0) return EPIC_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  int want = std::min(B, sm_count() * 2);
+  epic_status s = ensure_workspace(t, want, st);
+  if (s != EPIC_OK) return s;
+  t->last = st;
+  int ctas = std::min(B, t->ctas);
+  k_select<<<ctas, kThreads, 0, st>>>(g->dg, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_tok, d_conf, d_selected,
+                                      pack_of(t), t->d_stats);
+  return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
+}
+
+epic_status epic_commit(int32_t* d_x, int32_t B, int32_t n, const int32_t* d_pos, int32_t k, const int32_t* d_tok,
+                        const uint8_t* d_selected, void* cuda_stream) {
+  if (B < 0 || n < 0 || k < 0) return EPIC_ERR_INVALID_ARG;
+  long long total = (long long)B * k;
+  if (total == 0) return EPIC_OK;
+  if (!d_x || !d_pos || !d_tok || !d_selected) return EPIC_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  k_commit<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(d_x, B, n, d_pos, k, d_tok, d_selected);
+  return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
+}
+
+epic_status epic_get_stats(const epic_lexer_table* t, epic_stats* out, size_t out_bytes, int reset) {
+  if (!t || !out || out_bytes < sizeof(epic_stats)) return EPIC_ERR_INVALID_ARG;
+  unsigned long long h[S_N];
+  if (cudaStreamSynchronize(t->last) != cudaSuccess) return EPIC_ERR_CUDA;
+  if (cudaMemcpy(h, t->d_stats, sizeof(h), cudaMemcpyDeviceToHost) != cudaSuccess) return EPIC_ERR_CUDA;
+  out->checks = h[S_CHECKS];
+  out->valid = h[S_VALID];
+  out->overflow = h[S_OVERFLOW];
+  out->bad_inputs = h[S_BAD];
+  out->columns = h[S_COLUMNS];
+  out->entries = h[S_ENTRIES];
+  out->cover_checks = h[S_COVER];
+  out->exact_checks = h[S_EXACT];
+  out->selected = h[S_SELECTED];
+  if (reset && cudaMemset(t->d_stats, 0, sizeof(h)) != cudaSuccess) return EPIC_ERR_CUDA;
+  return EPIC_OK;
+}
+
+}  // extern "C"

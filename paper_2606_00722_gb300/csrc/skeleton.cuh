@@ -1,0 +1,310 @@
+// The graph walk shared by exact recognition (EarleyCols) and the cover
+// group test (CoverCols): it enumerates the nodes of the partial-output graph
+// of x (+) Delta in topological order, building them from the lex table, and
+// asks the column type to combine, close and store each node.
+#pragma once
+#include "cover.cuh"
+#include "walk.cuh"
+
+namespace epic {
+
+template <class Cols>
+struct Walk {
+  Cols& cols;
+  const DevGrammar& g;
+  const LexEntry* table;
+  WalkScratch sc;
+  WalkShared& sh;
+  int vocab;
+
+  __device__ Walk(Cols& c, const DevGrammar& g_, const LexEntry* t, WalkScratch s, WalkShared& shared, int v)
+      : cols(c), g(g_), table(t), sc(s), sh(shared), vocab(v) {}
+
+  __device__ void label_set(const uint32_t* lbl8) {
+    for (int w = threadIdx.x; w < g.W; w += blockDim.x) {
+      uint32_t acc = 0;
+      for (int lw = 0; lw < 8; ++lw) {
+        uint32_t m = lbl8[lw];
+        while (m) {
+          int b = __ffs(m) - 1;
+          m &= m - 1;
+          int a = (lw << 5) + b;
+          if (a < g.T) acc |= g.exp_term[(size_t)a * g.W + w];
+        }
+      }
+      sh.lbl[w] = acc;
+    }
+    __syncthreads();
+  }
+  __device__ void label_one(int a) {
+    for (int w = threadIdx.x; w < g.W; w += blockDim.x) sh.lbl[w] = g.exp_term[(size_t)a * g.W + w];
+    __syncthreads();
+  }
+
+  __device__ static int token_at(const int32_t* x, const Subst& s, int i) {
+    for (int j = 0; j < s.n; ++j)
+      if (s.pos[j] == i) return s.tok[j];
+    return x[i];
+  }
+
+  // One token of a span: frontier (f_q lexer state, f_c column)[0..nf) ->
+  // new frontier.  Lexings from the same column with the same end state and
+  // the same terminals after the first share one path whose first edge
+  // carries all their first terminals.  Returns false on overflow.
+  __device__ bool span_step(int tok) {
+    int nf = sh.nf;
+    const LexEntry* row = table + (size_t)tok * g.Q;
+    for (int f = threadIdx.x; f < nf; f += blockDim.x) {
+      LexEntry e = row[sc.f_q[f]];
+      int src = sc.f_c[f];
+      int leader = -1;
+      if (e.end != 0xFFFF) {
+        leader = f;
+        for (int h = 0; h < f; ++h) {
+          if (sc.f_c[h] != src) continue;
+          LexEntry e2 = row[sc.f_q[h]];
+          if (e2.end != e.end || e2.len != e.len) continue;
+          bool same = true;
+          for (int t = 1; t < e.len; ++t) same &= e.term[t] == e2.term[t];
+          if (same) {
+            leader = h;
+            break;
+          }
+        }
+      }
+      sc.key_q[f] = leader;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int ng = 0;
+      for (int f = 0; f < nf; ++f) {
+        if (sc.key_q[f] != f) continue;
+        LexEntry e = row[sc.f_q[f]];
+        sc.g_src[ng] = sc.f_c[f];
+        sc.g_end[ng] = e.end;
+        sc.g_len[ng] = e.len;
+        for (int t = 0; t < 16; ++t) sc.g_tail[ng * 16 + t] = (t + 1 < e.len) ? e.term[t + 1] : 0;
+        for (int w = 0; w < 8; ++w) sc.g_lbl[ng * 8 + w] = 0;
+        sc.key_q[f] = -2 - ng;
+        ++ng;
+      }
+      for (int f = 0; f < nf; ++f) {
+        int k = sc.key_q[f];
+        if (k == -1) continue;
+        int gid = (k <= -2) ? (-2 - k) : (-2 - sc.key_q[k]);
+        LexEntry e = row[sc.f_q[f]];
+        if (e.len > 0) sc.g_lbl[gid * 8 + (e.term[0] >> 5)] |= 1u << (e.term[0] & 31);
+      }
+      sh.ng = ng;
+    }
+    __syncthreads();
+    int ng = sh.ng;
+    // the run up to its last terminal (intermediate nodes)
+    for (int gi = 0; gi < ng; ++gi) {
+      int len = sc.g_len[gi];
+      int cur = sc.g_src[gi];
+      for (int t = 0; t + 1 < len; ++t) {
+        int c = cols.open_column();
+        __syncthreads();
+        if (c < 0) return false;
+        if (t == 0)
+          label_set(sc.g_lbl + gi * 8);
+        else
+          label_one(sc.g_tail[gi * 16 + t - 1]);
+        cols.arrive_labels(cur, false);
+        cols.close_column(c, false);
+        cols.finish_column(c);
+        if (sh.status != kWalkOk) return false;
+        cur = c;
+      }
+      if (threadIdx.x == 0) sc.g_last[gi] = cur;
+      __syncthreads();
+    }
+    // one node per distinct end state, ascending
+    if (threadIdx.x == 0) {
+      int nt = 0;
+      for (int gi = 0; gi < ng; ++gi) {
+        int e = sc.g_end[gi];
+        bool seen = false;
+        for (int j = 0; j < nt; ++j) seen |= sc.f_q[j] == e;
+        if (!seen) sc.f_q[nt++] = e;
+      }
+      for (int i = 1; i < nt; ++i) {
+        int v = sc.f_q[i], j = i - 1;
+        while (j >= 0 && sc.f_q[j] > v) {
+          sc.f_q[j + 1] = sc.f_q[j];
+          --j;
+        }
+        sc.f_q[j + 1] = v;
+      }
+      sh.nt = nt;
+    }
+    __syncthreads();
+    int nt = sh.nt;
+    for (int ti = 0; ti < nt; ++ti) {
+      int e = sc.f_q[ti];
+      int c = cols.open_column();
+      __syncthreads();
+      if (c < 0) return false;
+      for (int gi = 0; gi < ng; ++gi) {
+        if (sc.g_end[gi] != e) continue;
+        int len = sc.g_len[gi];
+        if (len == 0) {
+          cols.arrive_labels(sc.g_src[gi], true);
+        } else if (len == 1) {
+          label_set(sc.g_lbl + gi * 8);
+          cols.arrive_labels(sc.g_src[gi], false);
+        } else {
+          label_one(sc.g_tail[gi * 16 + len - 2]);
+          cols.arrive_labels(sc.g_last[gi], false);
+        }
+      }
+      cols.close_column(c, false);
+      cols.finish_column(c);
+      if (sh.status != kWalkOk) return false;
+      if (threadIdx.x == 0) sc.f_c[ti] = c;
+      __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+      int k = 0;
+      for (int ti = 0; ti < nt; ++ti)
+        if (!cols.column_empty(sc.f_c[ti])) {
+          sc.f_q[k] = sc.f_q[ti];
+          sc.f_c[k] = sc.f_c[ti];
+          ++k;
+        }
+      sh.nf = k;
+    }
+    __syncthreads();
+    return true;
+  }
+
+  // Walk x (+) s.  Returns 1 (accept item at the accept node), 0, -1 on a
+  // capacity overflow, -2 on bad input (unmasked position, bad token id).
+  __device__ int run(const int32_t* x, int n, Subst s) {
+    cols.reset();
+    if (threadIdx.x == 0) {
+      for (int j = 0; j < s.n; ++j) {
+        int p = s.pos[j];
+        if (p < 0 || p >= n || x[p] >= 0 || s.tok[j] < 0 || s.tok[j] >= vocab) sh.status = kWalkBadInput;
+      }
+    }
+    __syncthreads();
+    if (sh.status != kWalkOk) return -2;
+    int r = run_inner(x, n, s);
+    if (r < 0) cols.cleanup();
+    return r;
+  }
+
+  __device__ int seed_column(bool gap) {
+    int c = cols.open_column();
+    __syncthreads();
+    if (c < 0) return -1;
+    if (threadIdx.x == 0) sh.start_col = c;
+    __syncthreads();
+    cols.seed(c);
+    return c;
+  }
+
+  __device__ int run_inner(const int32_t* x, int n, Subst s) {
+    if (n == 0) {
+      int c = seed_column(false);
+      if (c < 0) return -1;
+      cols.close_column(c, false);
+      cols.finish_column(c);
+      if (sh.status != kWalkOk) return -1;
+      return cols.column_has_accept(c, c) ? 1 : 0;
+    }
+    int i = 0;
+    bool first = true;
+    int prev_gap = -1;
+    while (i < n) {
+      int t0 = token_at(x, s, i);
+      int j = i;
+      if (t0 < 0) {
+        while (j < n && token_at(x, s, j) < 0) ++j;
+        int c;
+        if (first) {
+          c = seed_column(true);
+          if (c < 0) return -1;
+        } else {
+          c = cols.open_column();
+          __syncthreads();
+          if (c < 0) return -1;
+          // the span before the gap: a pending lexeme that some byte can
+          // extend stays open (the gap absorbs its terminal); one that no
+          // byte can extend has ended and emits its terminal
+          int nf = sh.nf;
+          for (int f = 0; f < nf; ++f) {
+            int q = sc.f_q[f];
+            int a = g.dfa_accept[q];
+            if (q == 0 || g.dfa_ext[q] || (a >= 0 && g.skip[a])) {
+              cols.arrive_labels(sc.f_c[f], true);
+            } else if (a >= 0) {
+              label_one(a);
+              cols.arrive_labels(sc.f_c[f], false);
+            }
+          }
+        }
+        cols.close_column(c, true);
+        cols.finish_column(c);
+        if (sh.status != kWalkOk) return -1;
+        prev_gap = c;
+        if (cols.column_empty(c)) return 0;
+      } else {
+        while (j < n && token_at(x, s, j) >= 0) ++j;
+        if (first) {
+          int c = seed_column(false);
+          if (c < 0) return -1;
+          cols.close_column(c, false);
+          cols.finish_column(c);
+          if (sh.status != kWalkOk) return -1;
+          if (threadIdx.x == 0) {
+            sc.f_q[0] = 0;
+            sc.f_c[0] = c;
+            sh.nf = 1;
+          }
+        } else {
+          for (int q = threadIdx.x; q < g.Q; q += blockDim.x) {
+            sc.f_q[q] = q;
+            sc.f_c[q] = prev_gap;
+          }
+          if (threadIdx.x == 0) sh.nf = g.Q;
+        }
+        __syncthreads();
+        for (int p = i; p < j; ++p) {
+          if (sh.nf == 0) break;
+          int tok = token_at(x, s, p);
+          if (tok < 0 || tok >= vocab) return -2;
+          if (!span_step(tok)) return -1;
+        }
+        if (sh.nf == 0) return 0;  // no lexing of this span survives
+        if (j == n) {              // END: flush the pending lexeme
+          int c = cols.open_column();
+          __syncthreads();
+          if (c < 0) return -1;
+          int nf = sh.nf;
+          for (int f = 0; f < nf; ++f) {
+            int q = sc.f_q[f];
+            int a = g.dfa_accept[q];
+            if (q == 0 || (a >= 0 && g.skip[a])) {
+              cols.arrive_labels(sc.f_c[f], true);
+            } else if (a >= 0) {
+              label_one(a);
+              cols.arrive_labels(sc.f_c[f], false);
+            }
+          }
+          cols.close_column(c, false);
+          cols.finish_column(c);
+          if (sh.status != kWalkOk) return -1;
+          return cols.column_has_accept(c, sh.start_col) ? 1 : 0;
+        }
+      }
+      first = false;
+      i = j;
+    }
+    return cols.column_has_accept(prev_gap, sh.start_col) ? 1 : 0;
+  }
+};
+
+}  // namespace epic

@@ -1,0 +1,234 @@
+"""Thin ctypes binding of the EPIC C-ABI (``include/epic.h``).
+
+Argument marshalling only: every step of the hot path runs in the CUDA
+library ``_build/libepic.so``.  Device buffers are passed as torch CUDA
+tensors (their data pointers), host buffers as numpy arrays.  If the library
+is missing or no CUDA device is usable the calls raise -- there is no CPU
+fallback.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = [os.path.join(_HERE, 'csrc', f) for f in ('epic.cu', 'grammar.cpp')]
+_DEPS = _SRC + [os.path.join(_HERE, 'csrc', f) for f in
+                ('grammar.h', 'device.cuh', 'walk.cuh', 'cover.cuh', 'skeleton.cuh')] + \
+    [os.path.join(_HERE, '..', 'include', 'epic.h')]
+LIB_PATH = os.path.join(_HERE, '_build', 'libepic.so')
+NVCC_FLAGS = ['-gencode', 'arch=compute_103a,code=sm_103a', '-lineinfo', '-O3', '-std=c++17',
+              '-shared', '-Xcompiler', '-fPIC']
+
+OK, ERR_INVALID_ARG, ERR_GRAMMAR, ERR_LEXER, ERR_OOM, ERR_CUDA, ERR_CAPACITY, ERR_TIMEOUT = range(8)
+
+
+class EpicError(RuntimeError):
+    def __init__(self, status, where):
+        super().__init__('%s: %s (status %d)' % (where, _status_string(status), status))
+        self.status = status
+
+
+def build(force: bool = False, verbose: bool = False) -> str:
+    """Compile the CUDA library for sm_103a (nvcc cross-compiles without a GPU)."""
+    os.makedirs(os.path.dirname(LIB_PATH), exist_ok=True)
+    newest = max(os.path.getmtime(p) for p in _DEPS)
+    if force or not os.path.exists(LIB_PATH) or os.path.getmtime(LIB_PATH) < newest:
+        tmp = LIB_PATH + '.tmp%d' % os.getpid()
+        cmd = ['nvcc'] + NVCC_FLAGS + _SRC + ['-o', tmp]
+        if verbose:
+            print(' '.join(cmd))
+        subprocess.check_call(cmd)
+        os.replace(tmp, LIB_PATH)
+    return LIB_PATH
+
+
+class _Stats(C.Structure):
+    _fields_ = [(n, C.c_uint64) for n in ('checks', 'valid', 'overflow', 'bad_inputs', 'columns',
+                                          'entries', 'cover_checks', 'exact_checks', 'selected')]
+
+
+class _Desc(C.Structure):
+    _fields_ = [('n_terminals', C.c_int32), ('terminal_regex', C.POINTER(C.c_char_p)),
+                ('terminal_skip', C.POINTER(C.c_uint8)), ('n_nonterminals', C.c_int32),
+                ('start', C.c_int32), ('n_productions', C.c_int32), ('lhs', C.POINTER(C.c_int32)),
+                ('rhs_off', C.POINTER(C.c_int32)), ('rhs', C.POINTER(C.c_int32))]
+
+
+_lib = None
+EXPORTS = ('epic_grammar_create', 'epic_grammar_destroy', 'epic_grammar_lexer_states',
+           'epic_lexer_table_build', 'epic_lexer_table_destroy', 'epic_lexer_table_copy',
+           'epic_validate_batch',
+           'epic_pick_candidates', 'epic_select_compatible_subset', 'epic_commit',
+           'epic_get_stats', 'epic_status_string')
+
+
+def load(path: str | None = None):
+    """Load the library (raises OSError if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    lib = C.CDLL(path or LIB_PATH)
+    vp, i32, u8p, i32p = C.c_void_p, C.c_int32, C.POINTER(C.c_uint8), C.POINTER(C.c_int32)
+    lib.epic_status_string.restype = C.c_char_p
+    lib.epic_status_string.argtypes = [C.c_int]
+    lib.epic_grammar_create.argtypes = [C.POINTER(_Desc), C.POINTER(vp)]
+    lib.epic_grammar_destroy.argtypes = [vp]
+    lib.epic_grammar_lexer_states.argtypes = [vp]
+    lib.epic_grammar_lexer_states.restype = i32
+    lib.epic_lexer_table_build.argtypes = [vp, i32p, u8p, i32, vp, C.POINTER(vp)]
+    lib.epic_lexer_table_destroy.argtypes = [vp]
+    lib.epic_lexer_table_copy.argtypes = [vp, i32, i32, vp, C.c_size_t]
+    lib.epic_validate_batch.argtypes = [vp, vp, vp, i32, i32, vp, i32, vp, i32, vp, vp]
+    lib.epic_pick_candidates.argtypes = [vp, vp, vp, i32, i32, i32, vp, vp, vp]
+    lib.epic_select_compatible_subset.argtypes = [vp, vp, vp, i32, i32, vp, i32, vp, vp, vp, vp]
+    lib.epic_commit.argtypes = [vp, i32, i32, vp, i32, vp, vp, vp]
+    lib.epic_get_stats.argtypes = [vp, C.POINTER(_Stats), C.c_size_t, C.c_int]
+    _lib = lib
+    return lib
+
+
+def _status_string(s):
+    try:
+        return load().epic_status_string(int(s)).decode()
+    except OSError:
+        return 'status %d' % s
+
+
+def _check(status, where):
+    if status != OK:
+        raise EpicError(status, where)
+
+
+def _ptr(t):
+    """Device pointer of a torch tensor (or an int address)."""
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    if not t.is_cuda:
+        raise ValueError('expected a CUDA tensor')
+    if not t.is_contiguous():
+        raise ValueError('expected a contiguous tensor')
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+class Grammar:
+    """epic_grammar_create / epic_grammar_destroy."""
+
+    def __init__(self, spec):
+        lib = load()
+        T = spec.T
+        self._regs = (C.c_char_p * T)(*[t.regex.encode('latin-1') for t in spec.terminals])
+        self._skip = np.array([1 if t.skip else 0 for t in spec.terminals], np.uint8)
+        lhs, off, rhs = spec.rhs_flat()
+        self._arrs = (lhs, off, rhs if rhs.size else np.zeros(1, np.int32))
+        d = _Desc(T, self._regs, self._skip.ctypes.data_as(C.POINTER(C.c_uint8)), spec.V, spec.start,
+                  len(spec.productions), lhs.ctypes.data_as(C.POINTER(C.c_int32)),
+                  off.ctypes.data_as(C.POINTER(C.c_int32)),
+                  self._arrs[2].ctypes.data_as(C.POINTER(C.c_int32)))
+        h = C.c_void_p()
+        _check(lib.epic_grammar_create(C.byref(d), C.byref(h)), 'epic_grammar_create')
+        self.h = h
+        self.spec = spec
+
+    @property
+    def lexer_states(self):
+        return load().epic_grammar_lexer_states(self.h)
+
+    def close(self):
+        if getattr(self, 'h', None):
+            load().epic_grammar_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class LexTable:
+    """epic_lexer_table_build / epic_lexer_table_destroy."""
+
+    def __init__(self, grammar: Grammar, vocab, stream=None):
+        lib = load()
+        lens = np.array([len(t) for t in vocab], np.int64)
+        off = np.zeros(len(vocab) + 1, np.int32)
+        off[1:] = np.cumsum(lens)
+        data = np.frombuffer(b''.join(vocab), np.uint8).copy()
+        h = C.c_void_p()
+        _check(lib.epic_lexer_table_build(grammar.h, off.ctypes.data_as(C.POINTER(C.c_int32)),
+                                          data.ctypes.data_as(C.POINTER(C.c_uint8)), len(vocab),
+                                          _stream(stream), C.byref(h)), 'epic_lexer_table_build')
+        self.h = h
+        self.grammar = grammar
+        self.vocab = len(vocab)
+
+    def entries(self, first: int = 0, count: int | None = None):
+        """Lex-table rows as (end [count][Q] uint16, len [count][Q] uint8,
+        terms [count][Q][13] uint8); end 0xFFFF is DEAD."""
+        count = self.vocab - first if count is None else count
+        Q = self.grammar.lexer_states
+        raw = np.zeros((count, Q, 16), np.uint8)
+        _check(load().epic_lexer_table_copy(self.h, first, count, raw.ctypes.data, raw.nbytes),
+               'epic_lexer_table_copy')
+        end = raw[:, :, 0].astype(np.uint16) | (raw[:, :, 1].astype(np.uint16) << 8)
+        return end, raw[:, :, 2], raw[:, :, 3:16]
+
+    def stats(self, reset: bool = False) -> dict:
+        s = _Stats()
+        _check(load().epic_get_stats(self.h, C.byref(s), C.sizeof(s), int(reset)), 'epic_get_stats')
+        return {n: int(getattr(s, n)) for n, _ in _Stats._fields_}
+
+    def close(self):
+        if getattr(self, 'h', None):
+            load().epic_lexer_table_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def validate_batch(g: Grammar, t: LexTable, x, pos, cand, valid, stream=None):
+    B, n = x.shape
+    k = pos.shape[1]
+    K = cand.shape[2]
+    _check(load().epic_validate_batch(g.h, t.h, _ptr(x), B, n, _ptr(pos), k, _ptr(cand), K, _ptr(valid),
+                                      _stream(stream)), 'epic_validate_batch')
+
+
+def pick_candidates(cand, cand_conf, valid, tok, conf, stream=None):
+    B, k, K = cand.shape
+    _check(load().epic_pick_candidates(_ptr(cand), _ptr(cand_conf), _ptr(valid), B, k, K, _ptr(tok),
+                                       _ptr(conf), _stream(stream)), 'epic_pick_candidates')
+
+
+def select_compatible_subset(g: Grammar, t: LexTable, x, pos, tok, conf, selected, stream=None):
+    B, n = x.shape
+    k = pos.shape[1]
+    _check(load().epic_select_compatible_subset(g.h, t.h, _ptr(x), B, n, _ptr(pos), k, _ptr(tok),
+                                                _ptr(conf), _ptr(selected), _stream(stream)),
+           'epic_select_compatible_subset')
+
+
+def commit(x, pos, tok, selected, stream=None):
+    B, n = x.shape
+    k = pos.shape[1]
+    _check(load().epic_commit(_ptr(x), B, n, _ptr(pos), k, _ptr(tok), _ptr(selected), _stream(stream)),
+           'epic_commit')

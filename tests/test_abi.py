@@ -1,0 +1,48 @@
+"""The C-ABI library builds for sm_103a, loads, and exports every entry point
+that include/*.h declares; without a GPU the calls fail loudly (no CPU
+fallback)."""
+import glob
+import os
+import re
+
+import pytest
+
+import paper_2606_00722_gb300 as epic
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    names = set()
+    for h in glob.glob(os.path.join(ROOT, 'include', '*.h')):
+        src = open(h).read()
+        src = re.sub(r'/\*.*?\*/', '', src, flags=re.S)
+        for m in re.finditer(r'^[A-Za-z_][\w \*]*?\b(epic_\w+)\s*\(', src, flags=re.M):
+            names.add(m.group(1))
+    return names
+
+
+def test_library_exports_every_declared_symbol():
+    path = epic.build()
+    lib = epic.load(path)
+    names = declared_functions()
+    assert len(names) >= 12
+    for n in sorted(names):
+        assert hasattr(lib, n), n
+    assert set(epic.EXPORTS) <= names
+
+
+def test_status_strings():
+    lib = epic.load(epic.build())
+    for s in range(8):
+        assert lib.epic_status_string(s)
+
+
+def test_no_cpu_fallback_without_gpu():
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip('a GPU is present')
+    from synth import grammar_for
+    with pytest.raises(epic.EpicError) as e:
+        epic.Grammar(grammar_for('expr-tiny'))
+    assert e.value.status == 5  # EPIC_ERR_CUDA

@@ -1,0 +1,92 @@
+"""GPU parity: the CUDA path (through the C-ABI) against the CPU oracle,
+element by element on the same seeded inputs.  Validity bits and selected
+sets are integer results, so the bar is bit-exact equality."""
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+from synth import make_workload
+
+pytestmark = pytest.mark.gpu
+NTHREADS = os.cpu_count() or 1
+
+
+def _dev(a, dev):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+
+
+def gpu_step(w, dev):
+    import torch
+    import paper_2606_00722_gb300 as epic
+    g = epic.Grammar(w.grammar)
+    t = epic.LexTable(g, w.vocab)
+    x = _dev(w.x, dev)
+    pos = _dev(w.pos, dev)
+    cand = _dev(w.cand, dev)
+    conf3 = _dev(w.conf, dev)
+    valid = torch.empty(w.cand.shape, dtype=torch.uint8, device=dev)
+    epic.validate_batch(g, t, x, pos, cand, valid)
+    tok = torch.empty(w.pos.shape, dtype=torch.int32, device=dev)
+    conf = torch.empty(w.pos.shape, dtype=torch.float32, device=dev)
+    epic.pick_candidates(cand, conf3, valid, tok, conf)
+    sel = torch.empty(w.pos.shape, dtype=torch.uint8, device=dev)
+    epic.select_compatible_subset(g, t, x, pos, tok, conf, sel)
+    epic.commit(x, pos, tok, sel)
+    torch.cuda.synchronize()
+    return dict(valid=valid.cpu().numpy(), tok=tok.cpu().numpy(), conf=conf.cpu().numpy(),
+                sel=sel.cpu().numpy(), x=x.cpu().numpy(), stats=t.stats(), table=t, grammar=g)
+
+
+CASES = [
+    ('expr-tiny', 42, {}), ('expr-tiny', 43, {}), ('expr-tiny', 44, {}),
+    ('json-schema', 42, dict(batch=4)), ('json-schema', 43, dict(batch=3, k=3)),
+    ('smiles-256', 42, dict(batch=6, k=4)), ('smiles-256', 44, dict(batch=2, k=16, K=4)),
+    ('clike-512', 42, dict(batch=1, k=2, K=4)),
+]
+
+
+@pytest.mark.parametrize('name,seed,kw', CASES)
+def test_step_parity(cuda, name, seed, kw):
+    w = make_workload(name, seed, **kw)
+    O = oracle.Oracle(w.grammar, w.vocab)
+    got = gpu_step(w, cuda)
+    ref_valid = O.validate_batch(w.x, w.pos, w.cand, nthreads=NTHREADS)
+    assert (got['valid'] != 2).all(), 'capacity overflow'
+    np.testing.assert_array_equal(got['valid'], ref_valid)
+    rtok, rconf = oracle.pick_candidates(ref_valid, w.cand, w.conf)
+    np.testing.assert_array_equal(got['tok'], rtok)
+    np.testing.assert_array_equal(got['conf'], rconf)
+    ref_sel = O.select(w.x, w.pos, rtok, rconf)
+    np.testing.assert_array_equal(got['sel'], ref_sel)
+    np.testing.assert_array_equal(got['x'], O.commit(w.x, w.pos, rtok, ref_sel))
+    assert got['stats']['checks'] == w.cand.size
+
+
+@pytest.mark.parametrize('name', ['expr-tiny', 'json-schema', 'smiles-256'])
+def test_lex_table_runs_match_oracle(cuda, name):
+    """Every token's run from the initial state, and the set of distinct runs
+    over all lexer states, equal the oracle's lexing of the token's bytes."""
+    w = make_workload(name, 42, batch=1, vocab_size=2000 if name != 'expr-tiny' else None)
+    import paper_2606_00722_gb300 as epic
+    g = epic.Grammar(w.grammar)
+    t = epic.LexTable(g, w.vocab)
+    end, ln, terms = t.entries()
+    O = oracle.Oracle(w.grammar, w.vocab)
+    nstates = O.n_lexer_states
+    rng = np.random.default_rng(0)
+    for tok in rng.choice(len(w.vocab), size=min(300, len(w.vocab)), replace=False):
+        text = w.vocab[tok]
+        r0 = O.lex(text, 0, run_only=True)
+        assert (r0 is None) == (end[tok, 0] == 0xFFFF)
+        if r0 is not None:
+            assert list(terms[tok, 0, :ln[tok, 0]]) == r0[0]
+        mine = {tuple(terms[tok, q, :ln[tok, q]]) for q in range(end.shape[1]) if end[tok, q] != 0xFFFF}
+        ref = set()
+        for q in range(nstates):
+            r = O.lex(text, q, run_only=True)
+            if r is not None:
+                ref.add(tuple(r[0]))
+        assert mine == ref, (text, mine ^ ref)
