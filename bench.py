@@ -1,0 +1,308 @@
+"""Benchmark of one denoising step's constraint work on GB300.
+
+A step = epic_validate_batch + epic_pick_candidates +
+epic_select_compatible_subset + epic_commit over one batch of the workload
+(every proposed (position, candidate) pair checked, the compatible subset
+selected and committed).  Prints one JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   (the CPU oracle on the same config)
+
+Multi-GPU (torchrun, one rank per GPU): replicas -- every rank runs its own
+seeded batch of the same shape; there is no data-path collective.
+"""
+import argparse
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+INT_PEAK_NOTE = '152 SMs x 128 int32 lanes x 2.07 GHz'
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument('--gpus', type=int, default=1)
+    ap.add_argument('--steps', type=int, default=5)
+    ap.add_argument('--warmup', type=int, default=3)
+    ap.add_argument('--workload', default='json-schema')
+    ap.add_argument('--impl', default='epic', choices=['epic', 'reference'])
+    ap.add_argument('--seed', type=int, default=42)
+    ap.add_argument('--cpu-seconds', type=float, default=15.0)
+    ap.add_argument('--no-cpu-baseline', action='store_true')
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get('RANK', '0'))
+    world = int(os.environ.get('WORLD_SIZE', '1'))
+    local = int(os.environ.get('LOCAL_RANK', '0'))
+    return rank, world, local
+
+
+def peaks():
+    p = os.path.join(ROOT, 'MEASURED_PEAKS.json')
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, 'measured'
+    return {'hbm_gbs': 6800.0, 'bf16_tflops': 1900.0, 'sm_max_mhz': 2070.0}, 'fallback'
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, 'gpurun_out', 'bench_clocks.csv')
+
+    def __enter__(self):
+        os.makedirs(os.path.dirname(self.path), exist_ok=True)
+        q = ('index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,'
+             'clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,'
+             'clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap')
+        try:
+            self.f = open(self.path, 'w')
+            self.proc = subprocess.Popen(['nvidia-smi', '-i', str(self.index), '--query-gpu=' + q,
+                                          '--format=csv,noheader,nounits', '-lms', '200'],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if not self.proc or not os.path.exists(self.path):
+            return {'sm_mhz': None, 'sm_max_mhz': None, 'reasons': ['unsampled']}
+        sm, mx, reasons = [], [], set()
+        names = ['hw_slowdown', 'hw_thermal_slowdown', 'sw_thermal_slowdown', 'sw_power_cap']
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(',')]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for nm, v in zip(names, parts[5:9]):
+                    if v.lower() == 'active':
+                        reasons.add(nm)
+        if not sm:
+            return {'sm_mhz': None, 'sm_max_mhz': None, 'reasons': ['unsampled']}
+        return {'sm_mhz': float(np.median(sm)), 'sm_max_mhz': max(mx), 'reasons': sorted(reasons),
+                'samples': len(sm)}
+
+
+def cpu_baseline(w, seconds):
+    """The oracle as it stands on the host cores, on a bounded sample of the
+    workload's checks (whole sequences, all their candidates, in order)."""
+    import oracle
+    O = oracle.Oracle(w.grammar, w.vocab)
+    cores = os.cpu_count() or 1
+    per_seq = w.k * w.K
+    t0 = time.perf_counter()
+    done = 0
+    b = 0
+    while b < w.B and (time.perf_counter() - t0) < seconds:
+        O.validate_batch(w.x[b:b + 1], w.pos[b:b + 1], w.cand[b:b + 1], nthreads=cores)
+        done += per_seq
+        b += 1
+    dt = time.perf_counter() - t0
+    return {'value': done / dt, 'unit': 'checks/s', 'cores': cores, 'kind': 'oracle',
+            'sample': '%d of %d sequences (%d checks), oracle validate_batch on %d threads, %.1f s'
+                      % (b, w.B, done, cores, dt)}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    from synth import make_workload
+    w = make_workload(args.workload, args.seed)
+    import oracle
+    O = oracle.Oracle(w.grammar, w.vocab)
+    cores = os.cpu_count() or 1
+    # each step: a bounded sample of the workload (one sequence, all its
+    # candidates), sized so the whole run stays within minutes
+    per_step = []
+    for s in range(args.warmup + args.steps):
+        b = s % w.B
+        t0 = time.perf_counter()
+        O.validate_batch(w.x[b:b + 1], w.pos[b:b + 1], w.cand[b:b + 1], nthreads=cores)
+        dt = time.perf_counter() - t0
+        if s >= args.warmup:
+            per_step.append(dt)
+    checks = w.k * w.K
+    v = checks / float(np.mean(per_step))
+    line = {'impl': 'reference', 'metric': 'candidate validity checks/sec', 'value': v, 'unit': 'checks/s',
+            'n_gpus': 1, 'steps': args.steps, 'warmup': args.warmup,
+            'ms_per_step': float(np.mean(per_step)) * 1e3, 'higher_is_better': True, 'scaling': 'weak',
+            'vs_baseline': None, 'dtype': 'int32', 'data': 'synthetic',
+            'config': {'workload': args.workload, 'batch': 1, 'seq_len': w.n, 'k': w.k, 'K': w.K,
+                       'note': 'one sequence of the batch per step'},
+            'cpu_baseline': {'value': v, 'unit': 'checks/s', 'cores': cores, 'kind': 'oracle',
+                             'sample': 'one sequence (%d checks) per step' % checks},
+            'e2e': {'value': v, 'unit': 'checks/s', 'h2d_bytes_per_step': 0, 'd2h_bytes_per_step': 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == 'reference':
+        return run_reference(args)
+    import torch
+    import torch.distributed as dist
+    rank, world, local = dist_env()
+    if world > 1:
+        dist.init_process_group('nccl')
+    torch.cuda.set_device(local)
+    dev = torch.device('cuda', local)
+    import paper_2606_00722_gb300 as epic
+    epic.build()
+    from synth import make_workload
+    w = make_workload(args.workload, args.seed + rank)
+    g = epic.Grammar(w.grammar)
+    t = epic.LexTable(g, w.vocab)
+    x0 = torch.from_numpy(w.x).to(dev)
+    x = x0.clone()
+    pos = torch.from_numpy(w.pos).to(dev)
+    cand = torch.from_numpy(w.cand).to(dev)
+    conf3 = torch.from_numpy(w.conf).to(dev)
+    valid = torch.empty(w.cand.shape, dtype=torch.uint8, device=dev)
+    tok = torch.empty(w.pos.shape, dtype=torch.int32, device=dev)
+    conf = torch.empty(w.pos.shape, dtype=torch.float32, device=dev)
+    sel = torch.empty(w.pos.shape, dtype=torch.uint8, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # > 129 MB L2
+    stream = torch.cuda.current_stream()
+    checks = w.B * w.k * w.K
+    launches_per_step = 4
+
+    def step(xbuf):
+        epic.validate_batch(g, t, xbuf, pos, cand, valid)
+        epic.pick_candidates(cand, conf3, valid, tok, conf)
+        epic.select_compatible_subset(g, t, xbuf, pos, tok, conf, sel)
+        epic.commit(xbuf, pos, tok, sel)
+
+    for _ in range(args.warmup):
+        x.copy_(x0)
+        step(x)
+    torch.cuda.synchronize()
+    t.stats(reset=True)
+    # ---- device-timed region: per-step events, L2 flushed before each step
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with Clocks(local) as clk:
+        for i in range(args.steps):
+            x.copy_(x0)
+            flush.fill_(i & 255)
+            ev[i][0].record(stream)
+            epic.validate_batch(g, t, x, pos, cand, valid)
+            ev[i][1].record(stream)
+            epic.pick_candidates(cand, conf3, valid, tok, conf)
+            epic.select_compatible_subset(g, t, x, pos, tok, conf, sel)
+            epic.commit(x, pos, tok, sel)
+            ev[i][2].record(stream)
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    step_ms = [a.elapsed_time(c) for a, b, c in ev]
+    val_ms = [a.elapsed_time(b) for a, b, c in ev]
+    st = t.stats()
+    ms = float(np.mean(step_ms))
+    vms = float(np.mean(val_ms))
+    if world > 1:
+        tt = torch.tensor([ms, vms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms, vms = float(tt[0]), float(tt[1])
+    total_checks = checks * world
+    value = total_checks / (ms / 1e3)
+    # ---- end to end through the public API with host buffers
+    hx = torch.from_numpy(w.x).pin_memory()
+    hpos = torch.from_numpy(w.pos).pin_memory()
+    hcand = torch.from_numpy(w.cand).pin_memory()
+    hconf = torch.from_numpy(w.conf).pin_memory()
+    hvalid = torch.empty(w.cand.shape, dtype=torch.uint8).pin_memory()
+    hsel = torch.empty(w.pos.shape, dtype=torch.uint8).pin_memory()
+    hxo = torch.empty(w.x.shape, dtype=torch.int32).pin_memory()
+    e2e_ms = []
+    for i in range(args.steps):
+        flush.fill_(i & 255)
+        a, c = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        x.copy_(hx, non_blocking=True)
+        pos.copy_(hpos, non_blocking=True)
+        cand.copy_(hcand, non_blocking=True)
+        conf3.copy_(hconf, non_blocking=True)
+        step(x)
+        hvalid.copy_(valid, non_blocking=True)
+        hsel.copy_(sel, non_blocking=True)
+        hxo.copy_(x, non_blocking=True)
+        c.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms.append(a.elapsed_time(c))
+    e2e_step = float(np.mean(e2e_ms))
+    h2d = w.x.nbytes + w.pos.nbytes + w.cand.nbytes + w.conf.nbytes
+    d2h = w.cand.size + w.pos.size + w.x.nbytes
+    # ---- roofline of the dominant kernel (k_validate): bit-parallel Earley
+    # word operations, 3 passes (predict, scan, complete) over every stored
+    # (node, origin) entry of W words per check
+    pk, pk_kind = peaks()
+    sm_max = pk.get('sm_max_mhz', 2070.0)
+    int_peak = 152 * 128 * sm_max * 1e6 / 1e12  # T word-ops/s
+    entries = st['entries']
+    word_ops = 3.0 * entries * g_words(g)
+    achieved = word_ops / (vms / 1e3) / 1e12 / max(1, args.steps)
+    roof = {'bound': 'alu', 'achieved': achieved, 'peak': int_peak, 'unit': 'T word-ops/s',
+            'frac': achieved / int_peak, 'traffic': None,
+            'peak_source': 'derived: %s (%s sm_max_mhz)' % (INT_PEAK_NOTE, pk_kind),
+            'kernel': 'k_validate', 'kernel_ms': vms}
+    line = {'metric': 'candidate validity checks/sec', 'value': value, 'unit': 'checks/s',
+            'n_gpus': world, 'steps': args.steps, 'warmup': args.warmup, 'ms_per_step': ms,
+            'higher_is_better': True, 'scaling': 'weak', 'vs_baseline': None, 'dtype': 'int32',
+            'data': 'synthetic',
+            'config': {'workload': args.workload, 'batch': w.B, 'seq_len': w.n, 'k': w.k, 'K': w.K,
+                       'vocab': len(w.vocab), 'l2': 'flushed: 256 MiB write before every step',
+                       'parallelism': 'replicas' if world > 1 else 'single'},
+            'step_latency_us': ms * 1e3, 'validate_checks_per_s': total_checks / (vms / 1e3),
+            'valid_fraction': st['valid'] / max(1, st['checks']), 'overflow': st['overflow'],
+            'gpu_launches': launches_per_step * args.steps,
+            'e2e': {'value': total_checks / (e2e_step / 1e3), 'unit': 'checks/s', 'h2d_bytes_per_step': int(h2d),
+                    'd2h_bytes_per_step': int(d2h)},
+            'roofline': roof, 'clocks': clk.summary()}
+    if rank == 0:
+        if world == 1 and not args.no_cpu_baseline:
+            line['cpu_baseline'] = cpu_baseline(w, args.cpu_seconds)
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def g_words(g):
+    """Item words per chart entry of the grammar (W = ceil(D / 32))."""
+    spec = g.spec
+    D = sum(len(r) + 1 for _, r in spec.productions) + 2
+    return (D + 31) // 32
+
+
+if __name__ == '__main__':
+    main()
