@@ -20,6 +20,7 @@ struct DevGrammar {
   const uint32_t* exp_term;       // [T][W]
   const uint32_t* exp_nt;         // [V][W]
   const uint32_t* any_nt;         // [W]
+  const uint32_t* any_term;       // [W]
   const uint32_t* next_any;       // [W] items with a next symbol (excluding S' items)
   const uint32_t* nullable_next;  // [W]
   const uint32_t* complete;       // [W]

@@ -12,6 +12,7 @@
 #include "../../include/epic.h"
 #include "grammar.h"
 #include "skeleton.cuh"
+#include "warpwalk.cuh"
 
 using namespace epic;
 
@@ -139,6 +140,113 @@ __global__ void __launch_bounds__(kThreads) k_validate(DevGrammar g, const LexEn
       atomicAdd(&stats[S_ENTRIES], (unsigned long long)sh.nent);
     }
     __syncthreads();
+  }
+}
+
+// shared-memory staging of one warp: rows, completed-NT sets, slot origins,
+// origin slots (16-byte multiple)
+__host__ __device__ inline size_t smem_per_warp(int nmax, int rmax, int W, int VW) {
+  size_t b = (size_t)rmax * W * 4 + (size_t)rmax * VW * 4 + (size_t)rmax * 4 + (size_t)rmax * 8 + (size_t)nmax * 2;
+  return (b + 15) & ~(size_t)15;
+}
+
+struct WPack {
+  char* base;
+  size_t per_warp;
+  int nmax;
+  long long emax;
+  int W, VW;
+  __device__ WWs carve(long long warp) const {
+    WWs ws;
+    char* p = base + per_warp * (size_t)warp;
+    auto take = [&](size_t bytes) {
+      char* r = p;
+      p += (bytes + 255) & ~(size_t)255;
+      return r;
+    };
+    ws.stage = (uint32_t*)take((size_t)nmax * W * 4);
+    ws.bdone = (uint32_t*)take((size_t)nmax * VW * 4);
+    ws.col_off = (int32_t*)take((size_t)(nmax + 1) * 4);
+    ws.f_q = (int32_t*)take(kWMaxQ * 4);
+    ws.f_c = (int32_t*)take(kWMaxQ * 4);
+    ws.g_src = (int32_t*)take(kWMaxQ * 4);
+    ws.g_end = (int32_t*)take(kWMaxQ * 4);
+    ws.g_len = (int32_t*)take(kWMaxQ * 4);
+    ws.g_last = (int32_t*)take(kWMaxQ * 4);
+    ws.g_tail = (uint32_t*)take(kWMaxQ * 16);
+    ws.g_lbl = (uint32_t*)take(kWMaxQ * 32);
+    ws.ssum = (uint32_t*)take((size_t)nmax * 8);
+    ws.org = (int32_t*)take((size_t)emax * 4);
+    ws.esum = (uint32_t*)take((size_t)emax * 8);
+    ws.bits = (uint32_t*)take((size_t)emax * W * 4);
+    return ws;
+  }
+};
+
+static size_t wbytes_per_warp(int nmax, long long emax, int W, int VW) {
+  auto r = [](size_t b) { return (b + 255) & ~(size_t)255; };
+  return r((size_t)nmax * W * 4) + r((size_t)nmax * VW * 4) + r((size_t)(nmax + 1) * 4) + 6 * r(kWMaxQ * 4) +
+         r(kWMaxQ * 16) + r(kWMaxQ * 32) + r((size_t)nmax * 8) + r((size_t)emax * 4) + r((size_t)emax * 8) +
+         r((size_t)emax * W * 4);
+}
+
+// K2-K4 (warp form): one warp per validity check; warps pull checks from a
+// counter.  Each check walks the lexeme graph of x (+) (pos, tok) and runs
+// bit-parallel Earley recognition over it.
+template <bool SM>
+__global__ void __launch_bounds__(32 * kWarpsPerCta) k_validate_warp(
+    DevGrammar g, const LexEntry* __restrict__ table, int vocab, const int32_t* __restrict__ x, int n,
+    const int32_t* __restrict__ pos, int k, const int32_t* __restrict__ cand, int K, long long total,
+    uint8_t* __restrict__ valid, WPack wp, int rmax, unsigned long long* counter, unsigned long long* stats) {
+  __shared__ WSh shm[kWarpsPerCta];
+  extern __shared__ __align__(16) unsigned char dyn[];
+  int warp = threadIdx.x >> 5;
+  WSh& sh = shm[warp];
+  for (int w = threadIdx.x & 31; w < kWCols / 32; w += 32) {
+    sh.touched[w] = 0;
+    sh.dirty[w] = 0;
+  }
+  for (int v = threadIdx.x & 31; v < kWMaxVW; v += 32) {
+    sh.vset[v] = 0;
+    sh.vdone[v] = 0;
+  }
+  __syncwarp();
+  WarpWalker<SM> walk(g, table, wp.carve((long long)blockIdx.x * (blockDim.x >> 5) + warp), sh, wp.nmax, wp.emax,
+                      vocab);
+  if constexpr (SM) {
+    size_t per = smem_per_warp(wp.nmax, rmax, g.W, g.VW);
+    unsigned char* base = dyn + per * warp;
+    uint32_t* rows = (uint32_t*)base;
+    uint32_t* bd = rows + (size_t)rmax * g.W;
+    int32_t* sorg = (int32_t*)(bd + (size_t)rmax * g.VW);
+    uint32_t* ssum = (uint32_t*)(sorg + rmax);
+    int16_t* so = (int16_t*)(ssum + 2 * rmax);
+    walk.set_smem(rows, bd, so, sorg, ssum, rmax);
+  }
+  unsigned long long n_checks = 0, n_valid = 0, n_ovf = 0, n_bad = 0, n_cols = 0, n_ent = 0;
+  for (;;) {
+    long long jb = 0;
+    if ((threadIdx.x & 31) == 0) jb = (long long)atomicAdd(counter, 1ull);
+    jb = __shfl_sync(0xffffffffu, jb, 0);
+    if (jb >= total) break;
+    long long b = jb / ((long long)k * K);
+    long long j = (jb / K) % k;
+    int r = walk.run(x + b * n, n, pos[b * k + j], cand[jb]);
+    if ((threadIdx.x & 31) == 0) valid[jb] = r == 1 ? 1 : (r == -1 ? 2 : 0);
+    ++n_checks;
+    n_valid += r == 1;
+    n_ovf += r == -1;
+    n_bad += r == -2;
+    n_cols += walk.ncols;
+    n_ent += walk.nent;
+  }
+  if ((threadIdx.x & 31) == 0 && n_checks) {
+    atomicAdd(&stats[S_CHECKS], n_checks);
+    atomicAdd(&stats[S_VALID], n_valid);
+    atomicAdd(&stats[S_OVERFLOW], n_ovf);
+    atomicAdd(&stats[S_BAD], n_bad);
+    atomicAdd(&stats[S_COLUMNS], n_cols);
+    atomicAdd(&stats[S_ENTRIES], n_ent);
   }
 }
 
@@ -401,6 +509,11 @@ struct epic_lexer_table {
   int ctas = 0;
   unsigned long long* d_stats = nullptr;
   unsigned long long* d_counter = nullptr;
+  char* d_wws = nullptr;   // warp-walk workspace
+  size_t wws_bytes = 0;
+  int wnmax = 0;
+  long long wemax = 0;
+  int wwarps = 0;
   cudaStream_t last = nullptr;
 };
 
@@ -426,10 +539,10 @@ int sm_count() {
 }
 
 // Workspace sizing: columns <= 4096 per walk, entries as many as the budget
-// allows for the CTA count.  EPIC_WORKSPACE_MB (default 8192) caps the total.
+// allows for the CTA count.  EPIC_WORKSPACE_MB (default 2048) caps the total.
 epic_status ensure_workspace(epic_lexer_table* t, int want_ctas, cudaStream_t st) {
   const epic_grammar* g = t->g;
-  size_t budget_mb = 8192;
+  size_t budget_mb = 2048;
   if (const char* e = getenv("EPIC_WORKSPACE_MB")) budget_mb = strtoull(e, nullptr, 10);
   int W = g->dg.W, VW = g->dg.VW, FW = g->dg.FW;
   WsDims d;
@@ -472,6 +585,54 @@ epic_status ensure_workspace(epic_lexer_table* t, int want_ctas, cudaStream_t st
   return EPIC_OK;
 }
 
+// Warp-walk workspace: columns <= min(4096, 8 n + 256) per walk; entries
+// per walk EPIC_ENTRIES_PER_WALK (default 256 n); warps cut down until the
+// total fits EPIC_WARP_WORKSPACE_MB (default 6144).
+epic_status ensure_wworkspace(epic_lexer_table* t, long long checks, int n, cudaStream_t st) {
+  const epic_grammar* g = t->g;
+  int W = g->dg.W, VW = g->dg.VW;
+  int nmax = std::min(kWCols, 8 * n + 256);
+  long long emax = 256ll * std::max(1, n);
+  if (const char* e = getenv("EPIC_ENTRIES_PER_WALK")) emax = atoll(e);
+  size_t budget = (size_t)6144 << 20;
+  if (const char* e = getenv("EPIC_WARP_WORKSPACE_MB")) budget = strtoull(e, nullptr, 10) << 20;
+  size_t per = wbytes_per_warp(nmax, emax, W, VW);
+  long long warps = std::min<long long>(checks, (long long)sm_count() * 2 * kWarpsPerCta);
+  warps = std::max<long long>(kWarpsPerCta, (warps + kWarpsPerCta - 1) / kWarpsPerCta * kWarpsPerCta);
+  while (warps > kWarpsPerCta && per * (size_t)warps > budget) warps -= kWarpsPerCta;
+  size_t need = per * (size_t)warps;
+  if (t->d_wws && t->wws_bytes >= need && t->wnmax == nmax && t->wemax == emax) {
+    t->wwarps = (int)std::min<long long>(warps, t->wws_bytes / per / kWarpsPerCta * kWarpsPerCta);
+    return EPIC_OK;
+  }
+  if (t->d_wws) {
+    cudaStreamSynchronize(t->last);
+    cudaFree(t->d_wws);
+    t->d_wws = nullptr;
+  }
+  if (cudaMalloc(&t->d_wws, need) != cudaSuccess) {
+    t->d_wws = nullptr;
+    return EPIC_ERR_OOM;
+  }
+  if (cudaMemsetAsync(t->d_wws, 0, need, st) != cudaSuccess) return EPIC_ERR_CUDA;
+  t->wws_bytes = need;
+  t->wnmax = nmax;
+  t->wemax = emax;
+  t->wwarps = (int)warps;
+  return EPIC_OK;
+}
+
+WPack wpack_of(const epic_lexer_table* t) {
+  WPack p;
+  p.base = t->d_wws;
+  p.nmax = t->wnmax;
+  p.emax = t->wemax;
+  p.W = t->g->dg.W;
+  p.VW = t->g->dg.VW;
+  p.per_warp = wbytes_per_warp(p.nmax, p.emax, p.W, p.VW);
+  return p;
+}
+
 WsPack pack_of(const epic_lexer_table* t) {
   WsPack p;
   p.base = t->d_ws;
@@ -486,6 +647,19 @@ WsPack pack_of(const epic_lexer_table* t) {
 }  // namespace
 
 extern "C" {
+
+#ifdef EPIC_PHASE_TIMERS
+// measurement build only: per-phase cycle counters of the warp walker
+int epic_debug_phase_read(unsigned long long* out16, int reset) {
+  if (cudaDeviceSynchronize() != cudaSuccess) return -1;
+  if (cudaMemcpyFromSymbol(out16, g_phase, sizeof(unsigned long long) * 16) != cudaSuccess) return -1;
+  if (reset) {
+    unsigned long long z[16] = {0};
+    cudaMemcpyToSymbol(g_phase, z, sizeof(z));
+  }
+  return 0;
+}
+#endif
 
 const char* epic_status_string(epic_status s) {
   switch (s) {
@@ -582,6 +756,7 @@ epic_status epic_grammar_create(const epic_grammar_desc* desc, epic_grammar** ou
   up(G.exp_term, &d.exp_term);
   up(G.exp_nt, &d.exp_nt);
   up(G.any_nt, &d.any_nt);
+  up(G.any_term, &d.any_term);
   up(next_any, &d.next_any);
   up(G.nullable_next, &d.nullable_next);
   up(G.complete, &d.complete);
@@ -680,6 +855,7 @@ void epic_lexer_table_destroy(epic_lexer_table* t) {
   if (t->last) cudaStreamSynchronize(t->last);
   cudaFree(t->d_table);
   cudaFree(t->d_ws);
+  cudaFree(t->d_wws);
   cudaFree(t->d_stats);
   cudaFree(t->d_counter);
   delete t;
@@ -706,13 +882,31 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
   if (total == 0) return EPIC_OK;
   if (!d_x || !d_pos || !d_cand || !d_valid || n == 0) return EPIC_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)cuda_stream;
-  int want = (int)std::min<long long>(total, (long long)sm_count() * 2);
-  epic_status s = ensure_workspace(t, want, st);
+  epic_status s = ensure_wworkspace(t, total, n, st);
   if (s != EPIC_OK) return s;
   t->last = st;
   cudaMemsetAsync(t->d_counter, 0, 8, st);
-  k_validate<<<t->ctas, kThreads, 0, st>>>(g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total, d_valid,
-                                           pack_of(t), t->d_counter, t->d_stats);
+  // rows of the open column in shared memory (512 slots per warp, as many
+  // warps per CTA as fit) when the item set is narrow, else the global stage
+  WPack wp = wpack_of(t);
+  const size_t smem_cap = 190 * 1024;  // + 27 KB static per CTA <= 227 KB
+  const int rmax = 256;
+  size_t per = smem_per_warp(wp.nmax, rmax, wp.W, wp.VW);
+  int wpc = (int)std::min<size_t>(kWarpsPerCta, smem_cap / per);
+  if (const char* e = getenv("EPIC_GLOBAL_STAGE"))
+    if (atoi(e)) wpc = 0;
+  if (wp.W > 32) wpc = 0;
+  if (wpc >= 2) {
+    size_t dyn = per * wpc;
+    int blocks = t->wwarps / wpc;
+    cudaFuncSetAttribute(k_validate_warp<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+    k_validate_warp<true><<<blocks, 32 * wpc, dyn, st>>>(g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K,
+                                                          total, d_valid, wp, rmax, t->d_counter, t->d_stats);
+  } else {
+    k_validate_warp<false><<<t->wwarps / kWarpsPerCta, 32 * kWarpsPerCta, 0, st>>>(
+        g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total, d_valid, wp, 0, t->d_counter,
+        t->d_stats);
+  }
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
 }
 
