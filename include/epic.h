@@ -141,6 +141,35 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
                                 void* cuda_stream);
 
 /*
+ * epic_validate_batch without any device allocation.  The paper has no
+ * counterpart: this entry point is for callers that cannot call cudaMalloc
+ * -- a serving process that has handed all device memory to its own pool
+ * (model weights, KV cache) before decoding starts, or a per-step decode
+ * loop that must not take cudaMalloc's implicit device synchronization and
+ * unbounded latency.  Same arguments, outputs and errors as
+ * epic_validate_batch; results are identical.
+ *
+ * Scratch: a file-scope device array of 128 MiB inside the library, which
+ * every GPU that loads the library holds until the process exits.  Each
+ * walk needs (8 n + 256) columns and 256 n chart entries of workspace; if
+ * one walk's workspace does not fit in the array (long sequences with a
+ * wide grammar) the call returns EPIC_ERR_CAPACITY before enqueueing
+ * anything, and a check whose chart needs more than 256 n entries reports
+ * 2 (overflow) in d_valid.  Fewer walks run at once than in
+ * epic_validate_batch, so it is slower on large batches.
+ * The first call on a device looks up the array's device address (once per
+ * device, with that device current); make that first call before any
+ * stream capture.  Every call on a device shares the one array and keeps
+ * the last call's contents; the call clears what must start at zero.
+ * Calls that overlap on the GPU (on different streams, or from different
+ * threads) race on the array and must not be issued.
+ */
+epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_table* t,
+                                        const int32_t* d_x, int32_t B, int32_t n,
+                                        const int32_t* d_pos, int32_t k, const int32_t* d_cand,
+                                        int32_t K, uint8_t* d_valid, void* cuda_stream);
+
+/*
  * Candidate set C of Alg. 1 line 7 under the reading of the design notes:
  * per proposed position, the highest-confidence candidate whose valid bit is
  * 1 (ties: lowest candidate index), else none.  d_cand [B][k][K] int32,

@@ -4,6 +4,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <mutex>
 #include <new>
 #include <stdexcept>
 #include <string>
@@ -906,6 +907,81 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
     k_validate_warp<false><<<t->wwarps / kWarpsPerCta, 32 * kWarpsPerCta, 0, st>>>(
         g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total, d_valid, wp, 0, t->d_counter,
         t->d_stats);
+  }
+  return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
+}
+
+}  // extern "C"
+
+// ---------------------------------------------------------------- no-alloc validation
+// Scratch of epic_validate_batch_noalloc: a fixed device array that every GPU
+// which loads this library holds until the process exits.  Its first 256
+// bytes hold the work counter; the rest is carved into per-warp workspaces.
+constexpr size_t kNoAllocBytes = (size_t)128 << 20;
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
+
+namespace {
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[256] = {nullptr};  // device address of the array, per device ordinal
+}  // namespace
+
+extern "C" {
+
+epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_table* t, const int32_t* d_x,
+                                        int32_t B, int32_t n, const int32_t* d_pos, int32_t k,
+                                        const int32_t* d_cand, int32_t K, uint8_t* d_valid, void* cuda_stream) {
+  if (!g || !t || t->g != g || B < 0 || n < 0 || k < 0 || K < 0) return EPIC_ERR_INVALID_ARG;
+  long long total = (long long)B * k * K;
+  if (total == 0) return EPIC_OK;
+  if (!d_x || !d_pos || !d_cand || !d_valid || n == 0) return EPIC_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 256) return EPIC_ERR_CUDA;
+  char* base = nullptr;
+  {
+    // set-up, once per device, with that device current: host code may not
+    // use the array's name as a device address
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+      void* p = nullptr;
+      if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return EPIC_ERR_CUDA;
+      g_noalloc_ptr[dev] = p;
+    }
+    base = (char*)g_noalloc_ptr[dev];
+  }
+  const int W = g->dg.W, VW = g->dg.VW;
+  WPack wp;
+  wp.base = base + 256;
+  wp.nmax = std::min(kWCols, 8 * n + 256);
+  wp.emax = 256ll * n;
+  wp.W = W;
+  wp.VW = VW;
+  wp.per_warp = wbytes_per_warp(wp.nmax, wp.emax, W, VW);
+  long long fit = (long long)((kNoAllocBytes - 256) / wp.per_warp);
+  if (fit < 1) return EPIC_ERR_CAPACITY;  // one walk's workspace does not fit the array
+  const size_t smem_cap = 190 * 1024;
+  const int rmax = 256;
+  size_t sper = smem_per_warp(wp.nmax, rmax, W, VW);
+  int wpc = (W > 32) ? 0 : (int)std::min<size_t>(kWarpsPerCta, smem_cap / sper);
+  unsigned long long* counter = (unsigned long long*)base;
+  if (cudaMemsetAsync(counter, 0, sizeof(unsigned long long), st) != cudaSuccess) return EPIC_ERR_CUDA;
+  if (wpc >= 2) {
+    long long warps = std::min<long long>({total, fit, (long long)sm_count() * 2 * kWarpsPerCta});
+    int per_cta = (int)std::min<long long>(wpc, warps);
+    int blocks = (int)(warps / per_cta);
+    size_t dyn = sper * per_cta;
+    cudaFuncSetAttribute(k_validate_warp<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+    k_validate_warp<true><<<blocks, 32 * per_cta, dyn, st>>>(g->dg, t->d_table, t->vocab, d_x, n, d_pos, k,
+                                                              d_cand, K, total, d_valid, wp, rmax, counter,
+                                                              t->d_stats);
+  } else {
+    // the global stage and its completed-NT sets must start at zero
+    long long warps = std::min<long long>({total, fit, (long long)sm_count() * 2 * kWarpsPerCta});
+    int per_cta = (int)std::min<long long>(kWarpsPerCta, warps);
+    int blocks = (int)(warps / per_cta);
+    if (cudaMemsetAsync(wp.base, 0, wp.per_warp * (size_t)blocks * per_cta, st) != cudaSuccess) return EPIC_ERR_CUDA;
+    k_validate_warp<false><<<blocks, 32 * per_cta, 0, st>>>(g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand,
+                                                             K, total, d_valid, wp, 0, counter, t->d_stats);
   }
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
 }

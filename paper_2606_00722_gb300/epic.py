@@ -61,7 +61,7 @@ class _Desc(C.Structure):
 _lib = None
 EXPORTS = ('epic_grammar_create', 'epic_grammar_destroy', 'epic_grammar_lexer_states',
            'epic_lexer_table_build', 'epic_lexer_table_destroy', 'epic_lexer_table_copy',
-           'epic_validate_batch',
+           'epic_validate_batch', 'epic_validate_batch_noalloc',
            'epic_pick_candidates', 'epic_select_compatible_subset', 'epic_commit',
            'epic_get_stats', 'epic_status_string')
 
@@ -83,6 +83,7 @@ def load(path: str | None = None):
     lib.epic_lexer_table_destroy.argtypes = [vp]
     lib.epic_lexer_table_copy.argtypes = [vp, i32, i32, vp, C.c_size_t]
     lib.epic_validate_batch.argtypes = [vp, vp, vp, i32, i32, vp, i32, vp, i32, vp, vp]
+    lib.epic_validate_batch_noalloc.argtypes = [vp, vp, vp, i32, i32, vp, i32, vp, i32, vp, vp]
     lib.epic_pick_candidates.argtypes = [vp, vp, vp, i32, i32, i32, vp, vp, vp]
     lib.epic_select_compatible_subset.argtypes = [vp, vp, vp, i32, i32, vp, i32, vp, vp, vp, vp]
     lib.epic_commit.argtypes = [vp, i32, i32, vp, i32, vp, vp, vp]
@@ -211,6 +212,18 @@ def validate_batch(g: Grammar, t: LexTable, x, pos, cand, valid, stream=None):
     K = cand.shape[2]
     _check(load().epic_validate_batch(g.h, t.h, _ptr(x), B, n, _ptr(pos), k, _ptr(cand), K, _ptr(valid),
                                       _stream(stream)), 'epic_validate_batch')
+
+
+def validate_batch_noalloc(g: Grammar, t: LexTable, x, pos, cand, valid, stream=None):
+    """epic_validate_batch_noalloc: the same checks with no device allocation
+    (scratch in a fixed array inside the library), for callers whose device
+    memory is all reserved by their own pool or whose decode loop must not
+    call cudaMalloc.  Calls on one device must not overlap on the GPU."""
+    B, n = x.shape
+    k = pos.shape[1]
+    K = cand.shape[2]
+    _check(load().epic_validate_batch_noalloc(g.h, t.h, _ptr(x), B, n, _ptr(pos), k, _ptr(cand), K,
+                                              _ptr(valid), _stream(stream)), 'epic_validate_batch_noalloc')
 
 
 def pick_candidates(cand, cand_conf, valid, tok, conf, stream=None):
