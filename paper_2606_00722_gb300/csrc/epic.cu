@@ -194,11 +194,52 @@ static size_t wbytes_per_warp(int nmax, long long emax, int W, int VW) {
 // K2-K4 (warp form): one warp per validity check; warps pull checks from a
 // counter.  Each check walks the lexeme graph of x (+) (pos, tok) and runs
 // bit-parallel Earley recognition over it.
+// Bytes of the grammar tables the warp walk reads, staged in shared memory
+// (16-byte aligned pieces).
+__host__ __device__ inline size_t gtab_bytes(int T, int V, int W, int D, int Q) {
+  auto r = [](size_t b) { return (b + 15) & ~(size_t)15; };
+  return r((size_t)T * W * 4) + 2 * r((size_t)V * W * 4) + r((size_t)V * W * 4) + 5 * r((size_t)W * 4) +
+         2 * r((size_t)D * 2) + r((size_t)Q * 2) + r((size_t)Q) + r((size_t)T);
+}
+
+// Copy the walk's grammar tables into shared memory and point `out` at them.
+__device__ void stage_grammar(const DevGrammar& g, unsigned char* smem, DevGrammar& out) {
+  out = g;
+  unsigned char* p = smem;
+  auto put = [&](const void* src, size_t bytes) -> void* {
+    void* dst = p;
+    const uint32_t* s4 = (const uint32_t*)src;
+    uint32_t* d4 = (uint32_t*)dst;
+    size_t n4 = bytes / 4;
+    for (size_t i = threadIdx.x; i < n4; i += blockDim.x) d4[i] = s4[i];
+    for (size_t i = n4 * 4 + threadIdx.x; i < bytes; i += blockDim.x)
+      ((unsigned char*)dst)[i] = ((const unsigned char*)src)[i];
+    p += (bytes + 15) & ~(size_t)15;
+    return dst;
+  };
+  out.exp_term = (const uint32_t*)put(g.exp_term, (size_t)g.T * g.W * 4);
+  out.exp_nt = (const uint32_t*)put(g.exp_nt, (size_t)g.V * g.W * 4);
+  out.pred = (const uint32_t*)put(g.pred, (size_t)g.V * g.W * 4);
+  out.gap_pred = (const uint32_t*)put(g.gap_pred, (size_t)g.V * g.W * 4);
+  out.any_nt = (const uint32_t*)put(g.any_nt, (size_t)g.W * 4);
+  out.any_term = (const uint32_t*)put(g.any_term, (size_t)g.W * 4);
+  out.next_any = (const uint32_t*)put(g.next_any, (size_t)g.W * 4);
+  out.nullable_next = (const uint32_t*)put(g.nullable_next, (size_t)g.W * 4);
+  out.complete = (const uint32_t*)put(g.complete, (size_t)g.W * 4);
+  out.item_next = (const int16_t*)put(g.item_next, (size_t)g.D * 2);
+  out.item_lhs = (const int16_t*)put(g.item_lhs, (size_t)g.D * 2);
+  out.dfa_accept = (const int16_t*)put(g.dfa_accept, (size_t)g.Q * 2);
+  out.dfa_ext = (const uint8_t*)put(g.dfa_ext, (size_t)g.Q);
+  out.skip = (const uint8_t*)put(g.skip, (size_t)g.T);
+  __syncthreads();
+}
+
 template <bool SM>
 __global__ void __launch_bounds__(32 * kWarpsPerCta) k_validate_warp(
     DevGrammar g, const LexEntry* __restrict__ table, int vocab, const int32_t* __restrict__ x, int n,
     const int32_t* __restrict__ pos, int k, const int32_t* __restrict__ cand, int K, long long total,
-    uint8_t* __restrict__ valid, WPack wp, int rmax, unsigned long long* counter, unsigned long long* stats) {
+    uint8_t* __restrict__ valid, WPack wp, int rmax, int gtab_smem, unsigned long long* counter,
+    unsigned long long* stats) {
   __shared__ WSh shm[kWarpsPerCta];
   extern __shared__ __align__(16) unsigned char dyn[];
   int warp = threadIdx.x >> 5;
@@ -212,11 +253,20 @@ __global__ void __launch_bounds__(32 * kWarpsPerCta) k_validate_warp(
     sh.vdone[v] = 0;
   }
   __syncwarp();
-  WarpWalker<SM> walk(g, table, wp.carve((long long)blockIdx.x * (blockDim.x >> 5) + warp), sh, wp.nmax, wp.emax,
+  // the grammar tables in shared memory when they fit (gtab > 0)
+  DevGrammar gs = g;
+  size_t gt = 0;
+  if constexpr (SM) {
+    if (gtab_smem) {
+      stage_grammar(g, dyn, gs);
+      gt = gtab_bytes(g.T, g.V, g.W, g.D, g.Q);
+    }
+  }
+  WarpWalker<SM> walk(gs, table, wp.carve((long long)blockIdx.x * (blockDim.x >> 5) + warp), sh, wp.nmax, wp.emax,
                       vocab);
   if constexpr (SM) {
     size_t per = smem_per_warp(wp.nmax, rmax, g.W, g.VW);
-    unsigned char* base = dyn + per * warp;
+    unsigned char* base = dyn + gt + per * warp;
     uint32_t* rows = (uint32_t*)base;
     uint32_t* bd = rows + (size_t)rmax * g.W;
     int32_t* sorg = (int32_t*)(bd + (size_t)rmax * g.VW);
@@ -893,19 +943,26 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
   const size_t smem_cap = 190 * 1024;  // + 27 KB static per CTA <= 227 KB
   const int rmax = 256;
   size_t per = smem_per_warp(wp.nmax, rmax, wp.W, wp.VW);
-  int wpc = (int)std::min<size_t>(kWarpsPerCta, smem_cap / per);
+  const DevGrammar& dg = g->dg;
+  size_t gt = gtab_bytes(dg.T, dg.V, dg.W, dg.D, dg.Q);
+  int gsm = (gt + 4 * per <= smem_cap) ? 1 : 0;  // tables in shared memory if 4 warps still fit
+  int wpc = (int)std::min<size_t>(kWarpsPerCta, (smem_cap - (gsm ? gt : 0)) / per);
   if (const char* e = getenv("EPIC_GLOBAL_STAGE"))
     if (atoi(e)) wpc = 0;
   if (wp.W > 32) wpc = 0;
+  // spread the walks over every SM: no more warps per CTA than walks per SM
+  int per_sm = (int)((t->wwarps + sm_count() - 1) / sm_count());
+  if (wpc > per_sm) wpc = std::max(2, per_sm);
   if (wpc >= 2) {
-    size_t dyn = per * wpc;
-    int blocks = t->wwarps / wpc;
+    size_t dyn = per * wpc + (gsm ? gt : 0);
+    int blocks = (t->wwarps + wpc - 1) / wpc;
+    if ((size_t)blocks * wpc > (size_t)t->wwarps) blocks = t->wwarps / wpc;
     cudaFuncSetAttribute(k_validate_warp<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
     k_validate_warp<true><<<blocks, 32 * wpc, dyn, st>>>(g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K,
-                                                          total, d_valid, wp, rmax, t->d_counter, t->d_stats);
+                                                          total, d_valid, wp, rmax, gsm, t->d_counter, t->d_stats);
   } else {
     k_validate_warp<false><<<t->wwarps / kWarpsPerCta, 32 * kWarpsPerCta, 0, st>>>(
-        g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total, d_valid, wp, 0, t->d_counter,
+        g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total, d_valid, wp, 0, 0, t->d_counter,
         t->d_stats);
   }
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
@@ -972,7 +1029,7 @@ epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_
     size_t dyn = sper * per_cta;
     cudaFuncSetAttribute(k_validate_warp<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
     k_validate_warp<true><<<blocks, 32 * per_cta, dyn, st>>>(g->dg, t->d_table, t->vocab, d_x, n, d_pos, k,
-                                                              d_cand, K, total, d_valid, wp, rmax, counter,
+                                                              d_cand, K, total, d_valid, wp, rmax, 0, counter,
                                                               t->d_stats);
   } else {
     // the global stage and its completed-NT sets must start at zero
@@ -981,7 +1038,7 @@ epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_
     int blocks = (int)(warps / per_cta);
     if (cudaMemsetAsync(wp.base, 0, wp.per_warp * (size_t)blocks * per_cta, st) != cudaSuccess) return EPIC_ERR_CUDA;
     k_validate_warp<false><<<blocks, 32 * per_cta, 0, st>>>(g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand,
-                                                             K, total, d_valid, wp, 0, counter, t->d_stats);
+                                                             K, total, d_valid, wp, 0, 0, counter, t->d_stats);
   }
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
 }
