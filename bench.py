@@ -231,11 +231,9 @@ def main():
     ms = float(np.mean(step_ms))
     vms = float(np.mean(val_ms))
     if world > 1:
-        tt = torch.tensor([ms, vms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms, vms = float(tt[0]), float(tt[1])
+        ms, vms = max_over_ranks([ms, vms], dev)
     total_checks = checks * world
-    value = total_checks / (ms / 1e3)
+    value = job_value(checks, world, ms)
     # ---- end to end through the public API with host buffers
     hx = torch.from_numpy(w.x).pin_memory()
     hpos = torch.from_numpy(w.pos).pin_memory()
@@ -295,6 +293,22 @@ def main():
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def max_over_ranks(values, device=None):
+    """Element-wise maximum over all ranks of the default process group (the
+    job's time is its slowest rank's)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor(values, dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.cpu()]
+
+
+def job_value(checks_per_rank, world, ms):
+    """Whole-job throughput: the checks all ranks processed over the slowest
+    rank's step time."""
+    return checks_per_rank * world / (ms / 1e3)
 
 
 def g_words(g):
