@@ -127,10 +127,12 @@ epic_status epic_lexer_table_copy(const epic_lexer_table* t, int32_t first_token
  * d_x [B][n] int32 (-1 = MASK); d_pos [B][k] int32, each a masked position of
  * its row; d_cand [B][k][K] int32 token ids; d_valid [B][k][K] uint8 output:
  * 0 invalid, 1 valid, 2 capacity overflow for that check (no result).
- * The partial-output graph follows the gap reading of the design notes: each
- * maximal run of masks is one gap with a Sigma_lex* self-loop, each maximal
- * run of tokens a span lexed from q0 at the sequence start and from every
- * lexer state after a gap, flushed at END.  Host-side errors:
+ * The partial-output graph: each maximal run of masks is one gap with a
+ * Sigma_lex* self-loop (any terminal string, the mask count ignored); each
+ * maximal run of tokens is a span lexed from q0 at the sequence start and
+ * from every lexer state after a gap; before a gap a pending lexeme that some
+ * byte could extend stays open (the gap absorbs it) and one that no byte can
+ * extend is emitted; the last span is flushed at END.  Host-side errors:
  * EPIC_ERR_INVALID_ARG for sizes < 0 or NULL pointers with non-empty sizes.
  * Device-side: an unmasked position or an out-of-range token id yields 0 for
  * that check and counts in stats.bad_inputs.  Asynchronous.
@@ -170,7 +172,7 @@ epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_
                                         int32_t K, uint8_t* d_valid, void* cuda_stream);
 
 /*
- * Candidate set C of Alg. 1 line 7 under the reading of the design notes:
+ * Candidate set C of Alg. 1 line 7 ("high-confidence candidates"), read as:
  * per proposed position, the highest-confidence candidate whose valid bit is
  * 1 (ties: lowest candidate index), else none.  d_cand [B][k][K] int32,
  * d_cand_conf [B][k][K] float32, d_valid [B][k][K] uint8; outputs d_tok [B][k]

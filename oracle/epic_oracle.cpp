@@ -11,9 +11,9 @@
 //   * the flattened recursive-transition-network regular cover      (Sec. 4.3, App. A.2, App. D.3)
 //   * relaxed compatible subset selection + exact shrink            (Alg. 4)
 //
-// Readings where the paper is silent (lexer rule, gap model, cover
-// flattening, tie-breaks) are the ones listed in the design notes; each is
-// restated where it is implemented below.
+// Where the paper is silent (lexer rule, gap model, cover flattening,
+// tie-breaks) a reading is taken; each is stated where it is implemented
+// below.
 //
 // Only tests, the smoke check and the benchmark's CPU-baseline leg may load
 // this library.  It shares no code, header or table with the CUDA path: it
@@ -822,7 +822,7 @@ int orc_valid(void* h, const int* x, int n, long long* items) {
 }
 
 // Chart census of the full (exhaustive) chart: items and distinct origins per
-// node (a measurement aid for tests and design notes).
+// node (a measurement aid).
 int orc_chart_census(void* h, const int* x, int n, long long* items, int* origins, uint8_t* gap, int cap) {
   Grammar& g = ((Oracle*)h)->g;
   LexMemo memo;
