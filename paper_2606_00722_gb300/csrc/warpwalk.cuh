@@ -63,9 +63,13 @@ __device__ unsigned long long g_phase[16];
 #endif
 
 // SM = true keeps the rows of the column under construction in shared memory
-// (slot-mapped, rmax rows); SM = false keeps them in the per-warp global stage.
+// (slot-mapped, rmax rows) and handles item sets of at most 32 words (one
+// word per lane); SM = false keeps them in the per-warp global stage and
+// handles up to kWMaxW words.
 template <bool SM>
 class WarpWalker {
+  static constexpr int KW = SM ? 1 : kWMaxW / 32;  // item words per lane
+
  public:
   // shared-memory staging (SM): rows [rmax][W], completed-NT sets [rmax][VW],
   // slot of each origin (-1 = none) and origin of each slot
@@ -194,7 +198,6 @@ class WarpWalker {
   // row |= shift(row & M), until stable (item (p, d) -> (p, d+1)); the row is
   // held in registers (lane l owns words l, l+32, ...) while it is iterated
   __device__ void row_advance(uint32_t* row, const uint32_t* M) {
-    constexpr int KW = kWMaxW / 32;
     const int nw = (W + 31) >> 5;
     const int lane = wl_lane();
     uint32_t r[KW], m[KW];
