@@ -192,7 +192,7 @@ def main():
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # > 129 MB L2
     stream = torch.cuda.current_stream()
     checks = w.B * w.k * w.K
-    launches_per_step = 4
+    launches_per_step = 5  # validate, pick, select_spec, select, commit
 
     def step(xbuf):
         epic.validate_batch(g, t, xbuf, pos, cand, valid)

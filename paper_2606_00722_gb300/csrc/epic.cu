@@ -333,12 +333,61 @@ struct SelFrame {
   unsigned long long base, set, a, b;
 };
 
+// Alg. 4 always starts with the cover test of x (+) C and, when that passes,
+// continues with the exact test of the same x (+) C.  Both are run here at
+// once, one CTA each per sequence, before the recursion; k_select reuses the
+// two answers when it asks for exactly these tests.  spec[b] = {cover,
+// exact}: 1 pass, 0 fail, -1 not available (overflow / bad input).
+__global__ void __launch_bounds__(kThreads) k_select_spec(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
+                                                          const int32_t* __restrict__ x, int B, int n,
+                                                          const int32_t* __restrict__ pos, int k,
+                                                          const int32_t* __restrict__ tok, int8_t* __restrict__ spec,
+                                                          WsPack wsp) {
+  __shared__ WalkShared sh;
+  __shared__ int s_pos[kMaxSel], s_tok[kMaxSel];
+  __shared__ int ns;
+  Workspace ws;
+  WalkScratch sc;
+  wsp.carve(blockIdx.x, ws, sc);
+  for (int job = blockIdx.x; job < 2 * B; job += gridDim.x) {
+    int b = job >> 1;
+    bool exact = job & 1;
+    if (threadIdx.x == 0) {
+      int m = 0;
+      for (int j = 0; j < k; ++j) {
+        int t = tok[(long long)b * k + j];
+        if (t < 0) continue;
+        s_pos[m] = pos[(long long)b * k + j];
+        s_tok[m] = t;
+        ++m;
+      }
+      ns = m;
+    }
+    __syncthreads();
+    int r = -1;
+    if (ns >= 2) {  // a set of at most one candidate is never tested
+      Subst s{s_pos, s_tok, ns};
+      if (exact) {
+        EarleyCols cols(g, table, ws, sc, wsp.dims, sh);
+        Walk<EarleyCols> w(cols, g, table, sc, sh, vocab);
+        r = w.run(x + (long long)b * n, n, s);
+      } else {
+        CoverCols cols(g, ws, wsp.dims, sh);
+        Walk<CoverCols> w(cols, g, table, sc, sh, vocab);
+        r = w.run(x + (long long)b * n, n, s);
+      }
+    }
+    if (threadIdx.x == 0) spec[2 * b + (exact ? 1 : 0)] = (int8_t)(r == 1 ? 1 : (r == 0 ? 0 : -1));
+    __syncthreads();
+  }
+}
+
 __global__ void __launch_bounds__(kThreads) k_select(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
                                                      const int32_t* __restrict__ x, int B, int n,
                                                      const int32_t* __restrict__ pos, int k,
                                                      const int32_t* __restrict__ tok, const float* __restrict__ conf,
                                                      uint8_t* __restrict__ selected, WsPack wsp,
-                                                     unsigned long long* stats) {
+                                                     const int8_t* __restrict__ spec, unsigned long long* stats) {
   __shared__ WalkShared sh;
   __shared__ int c_slot[kMaxSel], c_pos[kMaxSel], c_tok[kMaxSel];
   __shared__ int s_pos[kMaxSel], s_tok[kMaxSel];
@@ -502,8 +551,11 @@ __global__ void __launch_bounds__(kThreads) k_select(DevGrammar g, const LexEntr
       int act = action;
       if (act == 0) break;
       Subst s{s_pos, s_tok, result};
+      // the test of the whole candidate set was run ahead (k_select_spec)
+      unsigned long long full = nc == 64 ? ~0ull : ((1ull << nc) - 1);
+      int cached = (spec && stack[sp - 1].a == full) ? spec[2 * b + (act == 1 ? 0 : 1)] : -1;
       __syncthreads();
-      int r = (act == 1) ? cover.run(xb, n, s) : exact.run(xb, n, s);
+      int r = cached >= 0 ? cached : ((act == 1) ? cover.run(xb, n, s) : exact.run(xb, n, s));
       if (threadIdx.x == 0) {
         if (r < 0) {
           overflow |= (r == -1);
@@ -560,6 +612,8 @@ struct epic_lexer_table {
   int ctas = 0;
   unsigned long long* d_stats = nullptr;
   unsigned long long* d_counter = nullptr;
+  int8_t* d_spec = nullptr;  // speculative Alg. 4 answers, 2 per sequence
+  int spec_cap = 0;
   char* d_wws = nullptr;   // warp-walk workspace
   size_t wws_bytes = 0;
   int wnmax = 0;
@@ -907,6 +961,7 @@ void epic_lexer_table_destroy(epic_lexer_table* t) {
   cudaFree(t->d_table);
   cudaFree(t->d_ws);
   cudaFree(t->d_wws);
+  cudaFree(t->d_spec);
   cudaFree(t->d_stats);
   cudaFree(t->d_counter);
   delete t;
@@ -1063,13 +1118,24 @@ epic_status epic_select_compatible_subset(const epic_grammar* g, const epic_lexe
   if ((long long)B * k == 0) return EPIC_OK;
   if (!d_x || !d_pos || !d_tok || !d_conf || !d_selected || n == 0) return EPIC_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)cuda_stream;
-  int want = std::min(B, sm_count() * 2);
+  int want = std::min(2 * B, sm_count() * 2);
   epic_status s = ensure_workspace(t, want, st);
   if (s != EPIC_OK) return s;
+  if (t->spec_cap < B) {
+    if (t->d_spec) {
+      cudaStreamSynchronize(t->last);
+      cudaFree(t->d_spec);
+    }
+    t->d_spec = nullptr;
+    if (cudaMalloc(&t->d_spec, (size_t)2 * B) != cudaSuccess) return EPIC_ERR_OOM;
+    t->spec_cap = B;
+  }
   t->last = st;
+  k_select_spec<<<std::min(2 * B, t->ctas), kThreads, 0, st>>>(g->dg, t->d_table, t->vocab, d_x, B, n, d_pos, k,
+                                                              d_tok, t->d_spec, pack_of(t));
   int ctas = std::min(B, t->ctas);
   k_select<<<ctas, kThreads, 0, st>>>(g->dg, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_tok, d_conf, d_selected,
-                                      pack_of(t), t->d_stats);
+                                      pack_of(t), t->d_spec, t->d_stats);
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
 }
 
