@@ -36,6 +36,7 @@ def parse():
     ap.add_argument('--seed', type=int, default=42)
     ap.add_argument('--cpu-seconds', type=float, default=15.0)
     ap.add_argument('--no-cpu-baseline', action='store_true')
+    ap.add_argument('--k', type=int, default=None, help='proposed positions per sequence (sweep)')
     return ap.parse_args()
 
 
@@ -135,7 +136,7 @@ def run_reference(args):
     if rank != 0:
         return
     from synth import make_workload
-    w = make_workload(args.workload, args.seed)
+    w = make_workload(args.workload, args.seed, k=args.k)
     import oracle
     O = oracle.Oracle(w.grammar, w.vocab)
     cores = os.cpu_count() or 1
@@ -155,10 +156,11 @@ def run_reference(args):
             'n_gpus': 1, 'steps': args.steps, 'warmup': args.warmup,
             'ms_per_step': float(np.mean(per_step)) * 1e3, 'higher_is_better': True, 'scaling': 'weak',
             'vs_baseline': None, 'dtype': 'int32', 'data': 'synthetic',
-            'config': {'workload': args.workload, 'batch': 1, 'seq_len': w.n, 'k': w.k, 'K': w.K,
-                       'note': 'one sequence of the batch per step'},
+            'config': {'workload': args.workload, 'batch': w.B, 'seq_len': w.n, 'k': w.k, 'K': w.K,
+                       'vocab': len(w.vocab), 'l2': 'n/a (host cores)', 'parallelism': 'single'},
             'cpu_baseline': {'value': v, 'unit': 'checks/s', 'cores': cores, 'kind': 'oracle',
-                             'sample': 'one sequence (%d checks) per step' % checks},
+                             'sample': 'one sequence of the batch (%d checks) per step, oracle validate_batch '
+                                       'on %d threads' % (checks, cores)},
             'e2e': {'value': v, 'unit': 'checks/s', 'h2d_bytes_per_step': 0, 'd2h_bytes_per_step': 0}}
     print(json.dumps(line), flush=True)
 
@@ -177,7 +179,7 @@ def main():
     import paper_2606_00722_gb300 as epic
     epic.build()
     from synth import make_workload
-    w = make_workload(args.workload, args.seed + rank)
+    w = make_workload(args.workload, args.seed + rank, k=args.k)
     g = epic.Grammar(w.grammar)
     t = epic.LexTable(g, w.vocab)
     x0 = torch.from_numpy(w.x).to(dev)
