@@ -275,7 +275,7 @@ def main():
     roof = {'bound': 'alu', 'achieved': achieved, 'peak': int_peak, 'unit': 'T word-ops/s',
             'frac': achieved / int_peak, 'traffic': None,
             'peak_source': 'derived: %s (%s sm_max_mhz)' % (INT_PEAK_NOTE, pk_kind),
-            'kernel': 'k_validate', 'kernel_ms': vms}
+            'kernel': 'k_validate_warp', 'kernel_ms': vms}
     line = {'metric': 'candidate validity checks/sec', 'value': value, 'unit': 'checks/s',
             'n_gpus': world, 'steps': args.steps, 'warmup': args.warmup, 'ms_per_step': ms,
             'higher_is_better': True, 'scaling': 'weak', 'vs_baseline': None, 'dtype': 'int32',
