@@ -107,43 +107,6 @@ static size_t ws_bytes_per_cta(const WsDims& d, int W, int VW, int FW) {
 
 enum StatIdx { S_CHECKS, S_VALID, S_OVERFLOW, S_BAD, S_COLUMNS, S_ENTRIES, S_COVER, S_EXACT, S_SELECTED, S_N };
 
-// K2-K4: one CTA per validity check (persistent CTAs pull checks from a
-// counter).  Each check walks the lexeme graph of x (+) (pos, tok) and runs
-// bit-parallel Earley recognition over it.
-__global__ void __launch_bounds__(kThreads) k_validate(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
-                                                       const int32_t* __restrict__ x, int n, const int32_t* __restrict__ pos,
-                                                       int k, const int32_t* __restrict__ cand, int K, long long total,
-                                                       uint8_t* __restrict__ valid, WsPack wsp,
-                                                       unsigned long long* counter, unsigned long long* stats) {
-  __shared__ WalkShared sh;
-  __shared__ long long job;
-  Workspace ws;
-  WalkScratch sc;
-  wsp.carve(blockIdx.x, ws, sc);
-  EarleyCols cols(g, table, ws, sc, wsp.dims, sh);
-  Walk<EarleyCols> walk(cols, g, table, sc, sh, vocab);
-  for (;;) {
-    if (threadIdx.x == 0) job = (long long)atomicAdd(counter, 1ull);
-    __syncthreads();
-    long long jb = job;
-    if (jb >= total) break;
-    long long b = jb / ((long long)k * K);
-    long long j = (jb / K) % k;
-    Subst s{pos + b * k + j, cand + jb, 1};
-    int r = walk.run(x + b * n, n, s);
-    if (threadIdx.x == 0) {
-      valid[jb] = r == 1 ? 1 : (r == -1 ? 2 : 0);
-      atomicAdd(&stats[S_CHECKS], 1ull);
-      if (r == 1) atomicAdd(&stats[S_VALID], 1ull);
-      if (r == -1) atomicAdd(&stats[S_OVERFLOW], 1ull);
-      if (r == -2) atomicAdd(&stats[S_BAD], 1ull);
-      atomicAdd(&stats[S_COLUMNS], (unsigned long long)sh.ncols);
-      atomicAdd(&stats[S_ENTRIES], (unsigned long long)sh.nent);
-    }
-    __syncthreads();
-  }
-}
-
 // shared-memory staging of one warp: rows, completed-NT sets, slot origins,
 // origin slots (16-byte multiple)
 __host__ __device__ inline size_t smem_per_warp(int nmax, int rmax, int W, int VW) {

@@ -46,3 +46,22 @@ def test_no_cpu_fallback_without_gpu():
     with pytest.raises(epic.EpicError) as e:
         epic.Grammar(grammar_for('expr-tiny'))
     assert e.value.status == 5  # EPIC_ERR_CUDA
+
+
+def test_host_side_argument_errors():
+    """Argument errors are detected on the host, before any device work."""
+    import ctypes as C
+    lib = epic.load(epic.build())
+    out = C.c_void_p()
+    assert lib.epic_grammar_create(None, C.byref(out)) == 1
+    d = epic.epic._Desc()
+    d.n_terminals = 0  # no terminals
+    assert lib.epic_grammar_create(C.byref(d), C.byref(out)) == 1
+    # null objects and negative sizes
+    assert lib.epic_validate_batch(None, None, None, 1, 1, None, 1, None, 1, None, None) == 1
+    assert lib.epic_select_compatible_subset(None, None, None, 1, 1, None, 1, None, None, None, None) == 1
+    assert lib.epic_commit(None, -1, 1, None, 1, None, None, None) == 1
+    assert lib.epic_pick_candidates(None, None, None, 1, 1, 1, None, None, None) == 1
+    # empty batches are no-ops that touch nothing
+    assert lib.epic_commit(None, 0, 5, None, 3, None, None, None) == 0
+    assert lib.epic_pick_candidates(None, None, None, 0, 4, 4, None, None, None) == 0
