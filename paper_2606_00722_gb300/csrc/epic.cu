@@ -264,6 +264,8 @@ __global__ void __launch_bounds__(32 * kWarpsPerCta) k_validate_warp(
   }
 }
 
+#include "region.cuh"
+
 // Per proposed position: the highest-confidence candidate with valid bit 1.
 __global__ void k_pick(const int32_t* __restrict__ cand, const float* __restrict__ conf,
                        const uint8_t* __restrict__ valid, int B, int k, int K, int32_t* __restrict__ tok,
@@ -576,6 +578,10 @@ struct epic_lexer_table {
   unsigned long long* d_stats = nullptr;
   unsigned long long* d_counter = nullptr;
   int8_t* d_spec = nullptr;  // speculative Alg. 4 answers, 2 per sequence
+  char* d_seq = nullptr;     // per-sequence forward charts (region checks)
+  size_t seq_bytes = 0;
+  int32_t* d_regs = nullptr; // per-warp tables of region checks
+  size_t regs_bytes = 0;
   int spec_cap = 0;
   char* d_wws = nullptr;   // warp-walk workspace
   size_t wws_bytes = 0;
@@ -699,6 +705,121 @@ WPack wpack_of(const epic_lexer_table* t) {
   p.VW = t->g->dg.VW;
   p.per_warp = wbytes_per_warp(p.nmax, p.emax, p.W, p.VW);
   return p;
+}
+
+// Grow a device buffer owned by the table (synchronizing its last stream first).
+epic_status grow(epic_lexer_table* t, char** buf, size_t* have, size_t need) {
+  if (*buf && *have >= need) return EPIC_OK;
+  if (*buf) {
+    cudaStreamSynchronize(t->last);
+    cudaFree(*buf);
+    *buf = nullptr;
+    *have = 0;
+  }
+  if (cudaMalloc(buf, need) != cudaSuccess) {
+    *buf = nullptr;
+    return EPIC_ERR_OOM;
+  }
+  *have = need;
+  return EPIC_OK;
+}
+
+// Region checks: forward chart and good masks per sequence, then one warp per
+// check.  Capacities: EPIC_SEQ_ENTRIES (default 400 n) chart entries per
+// sequence, EPIC_SEQ_WORKSPACE_MB (default 81920) in total; checks of a
+// sequence whose chart does not fit walk their whole graph instead.
+epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const int32_t* d_x, int B, int n,
+                            const int32_t* d_pos, int k, const int32_t* d_cand, int K, uint8_t* d_valid,
+                            cudaStream_t st) {
+  const DevGrammar& dg = g->dg;
+  long long total = (long long)B * k * K;
+  SeqPack sp;
+  sp.nmax = std::min(1900, 8 * n + 256);
+  sp.n = n;
+  sp.W = dg.W;
+  sp.VW = dg.VW;
+  sp.edge_cap = 32 * sp.nmax;
+  sp.emax = 400ll * n;
+  if (const char* e = getenv("EPIC_SEQ_ENTRIES")) sp.emax = atoll(e);
+  size_t budget = (size_t)81920 << 20;
+  if (const char* e = getenv("EPIC_SEQ_WORKSPACE_MB")) budget = strtoull(e, nullptr, 10) << 20;
+  while (sp.emax > 4096 && sp.bytes() * (size_t)B > budget) sp.emax = sp.emax * 3 / 4;
+  sp.per_seq = sp.bytes();
+  epic_status s = grow(t, &t->d_seq, &t->seq_bytes, sp.per_seq * (size_t)B);
+  if (s != EPIC_OK) return s;
+  sp.base = t->d_seq;
+  // per-warp workspace of the checks: own columns after the chart's
+  WPack wp;
+  wp.nmax = kWCols;
+  // own entries: the region's columns and the rows carried after it
+  wp.emax = std::max(8192ll, 64ll * n);
+  if (const char* e = getenv("EPIC_ENTRIES_PER_WALK")) wp.emax = atoll(e);
+  wp.W = dg.W;
+  wp.VW = dg.VW;
+  wp.per_warp = wbytes_per_warp(wp.nmax, wp.emax, wp.W, wp.VW);
+  size_t wbudget = (size_t)6144 << 20;
+  if (const char* e = getenv("EPIC_WARP_WORKSPACE_MB")) wbudget = strtoull(e, nullptr, 10) << 20;
+  long long warps = std::min<long long>(total, (long long)sm_count() * 2 * kWarpsPerCta);
+  warps = std::max<long long>(1, warps);
+  while (warps > 1 && wp.per_warp * (size_t)warps > wbudget) warps = warps * 3 / 4;
+  size_t wneed = wp.per_warp * (size_t)warps;
+  if (!t->d_wws || t->wws_bytes < wneed || t->wnmax != wp.nmax || t->wemax != wp.emax) {
+    if (t->d_wws) {
+      cudaStreamSynchronize(t->last);
+      cudaFree(t->d_wws);
+      t->d_wws = nullptr;
+    }
+    if (cudaMalloc(&t->d_wws, wneed) != cudaSuccess) {
+      t->d_wws = nullptr;
+      return EPIC_ERR_OOM;
+    }
+    // the global stage starts at zero; walks return it zeroed
+    if (cudaMemsetAsync(t->d_wws, 0, wneed, st) != cudaSuccess) return EPIC_ERR_CUDA;
+    t->wws_bytes = wneed;
+    t->wnmax = wp.nmax;
+    t->wemax = wp.emax;
+  }
+  wp.base = t->d_wws;
+  s = grow(t, (char**)&t->d_regs, &t->regs_bytes, (size_t)warps * 3 * wp.nmax * 4);
+  if (s != EPIC_OK) return s;
+  t->last = st;
+  const size_t smem_cap = 190 * 1024;
+  const int rmax = 256;
+  bool sm = dg.W <= 32;
+  // 1. forward charts
+  {
+    int wpc = kWarpsPerCta;
+    size_t per = smem_per_warp(sp.nmax, rmax, dg.W, dg.VW);
+    if (sm) wpc = (int)std::min<size_t>(kWarpsPerCta, smem_cap / per);
+    if (sm && wpc >= 1) {
+      size_t dyn = per * wpc;
+      cudaFuncSetAttribute(k_forward<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+      k_forward<true><<<(B + wpc - 1) / wpc, 32 * wpc, dyn, st>>>(dg, t->d_table, t->vocab, d_x, B, n, sp, rmax);
+    } else {
+      k_forward<false><<<(B + kWarpsPerCta - 1) / kWarpsPerCta, 32 * kWarpsPerCta, 0, st>>>(
+          dg, t->d_table, t->vocab, d_x, B, n, sp, 0);
+    }
+  }
+  // 2. good masks
+  k_good<<<(B + kWarpsPerCta - 1) / kWarpsPerCta, 32 * kWarpsPerCta, 0, st>>>(dg, B, sp);
+  // 3. checks
+  cudaMemsetAsync(t->d_counter, 0, 8, st);
+  size_t per = smem_per_warp(wp.nmax, rmax, dg.W, dg.VW);
+  int wpc = sm ? (int)std::min<size_t>(kWarpsPerCta, smem_cap / per) : 0;
+  wpc = (int)std::min<long long>(wpc, warps);  // every launched warp owns an allocated workspace
+  if (wpc >= 1) {
+    int blocks = (int)std::max<long long>(1, warps / wpc);
+    size_t dyn = per * wpc;
+    cudaFuncSetAttribute(k_check<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+    k_check<true><<<blocks, 32 * wpc, dyn, st>>>(dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total, d_valid,
+                                                 sp, wp, t->d_regs, rmax, t->d_counter, t->d_stats);
+  } else {
+    int per_cta = (int)std::min<long long>(kWarpsPerCta, warps);
+    int blocks = (int)std::max<long long>(1, warps / per_cta);
+    k_check<false><<<blocks, 32 * per_cta, 0, st>>>(dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total,
+                                                    d_valid, sp, wp, t->d_regs, 0, t->d_counter, t->d_stats);
+  }
+  return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
 }
 
 WsPack pack_of(const epic_lexer_table* t) {
@@ -925,6 +1046,8 @@ void epic_lexer_table_destroy(epic_lexer_table* t) {
   cudaFree(t->d_ws);
   cudaFree(t->d_wws);
   cudaFree(t->d_spec);
+  cudaFree(t->d_seq);
+  cudaFree(t->d_regs);
   cudaFree(t->d_stats);
   cudaFree(t->d_counter);
   delete t;
@@ -951,6 +1074,10 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
   if (total == 0) return EPIC_OK;
   if (!d_x || !d_pos || !d_cand || !d_valid || n == 0) return EPIC_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)cuda_stream;
+  // wide item sets (large grammars): checks by region over a per-sequence chart
+  bool region = g->dg.W > 32;
+  if (const char* e = getenv("EPIC_REGION")) region = atoi(e) != 0;
+  if (region) return validate_region(g, t, d_x, B, n, d_pos, k, d_cand, K, d_valid, st);
   epic_status s = ensure_wworkspace(t, total, n, st);
   if (s != EPIC_OK) return s;
   t->last = st;

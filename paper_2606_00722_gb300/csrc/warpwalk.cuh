@@ -40,6 +40,24 @@ struct WWs {  // per-warp global workspace
   uint32_t* g_lbl;   // [kWMaxQ][8]  first-terminal label set
 };
 
+// What a recording walk (a sequence's forward chart) writes besides the chart:
+// the graph's edges in creation order of their target, gap flags, where each
+// position's segment sits in the graph, and each entry's completed
+// nonterminals.
+struct SeqRec {
+  uint8_t* col_gap;    // [nmax]
+  int32_t* e_dst;      // [edge_cap]
+  int32_t* e_src;      // [edge_cap]
+  uint32_t* e_lbl;     // [edge_cap][8] terminal set of a labelled edge, all zero = epsilon
+  int32_t* gap_col;    // [n] masked position -> column of its gap
+  int32_t* pre_col;    // [n] fixed position -> column before its span (gap or BEGIN)
+  int32_t* post_col;   // [n] fixed position -> column after its span (gap or END)
+  uint32_t* cnt;       // [emax][VW] completed nonterminals of each entry
+  int32_t* meta;       // [8]: ncols, nedges, start, accept, status, nent (low), -, -
+  int edge_cap;
+  int n_edges;         // running count (kept by the walk)
+};
+
 struct WSh {  // per-warp shared memory
   uint32_t touched[kWCols / 32];
   uint32_t dirty[kWCols / 32];
@@ -95,6 +113,19 @@ class WarpWalker {
   int nf;
   int start_col;
   uint32_t label_fold = 0;  // bit (a mod 32) of every terminal in sh.lbl
+  // A read-only base chart (a sequence's forward chart) holds columns
+  // 0 .. base_cols-1 and entries 0 .. base_ent-1; this walk's own columns
+  // follow with ids from base_cols.
+  int base_cols = 0;
+  long long base_ent = 0;
+  const int32_t* b_col_off = nullptr;
+  const int32_t* b_org = nullptr;
+  const uint32_t* b_bits = nullptr;
+  const uint32_t* b_esum = nullptr;
+  // recording of the forward chart's graph (null when not recording)
+  SeqRec* rec = nullptr;
+  int cur_col = -1;
+  uint32_t cur_lbl8[8];      // label set of the arrivals being made (all zero = epsilon)
 
   __device__ WarpWalker(const DevGrammar& g_, const LexEntry* t, WWs w, WSh& s, int nm, long long em, int voc)
       : g(g_), table(t), ws(w), sh(s), nmax(nm), emax(em), vocab(voc), W(g_.W), VW(g_.VW) {}
@@ -151,6 +182,21 @@ class WarpWalker {
   __device__ uint32_t* sum_of(int o) {
     if constexpr (!SM) return ws.ssum + (size_t)o * 2;
     else return slot_sum + slot_of[o] * 2;
+  }
+
+  // ------------------------------------------------------------ chart access
+  __device__ long long cbeg(int c) const {
+    return c < base_cols ? (long long)b_col_off[c] : base_ent + ws.col_off[c - base_cols];
+  }
+  __device__ long long cend(int c) const {
+    return c < base_cols ? (long long)b_col_off[c + 1] : base_ent + ws.col_off[c - base_cols + 1];
+  }
+  __device__ int eorg(long long k) const { return k < base_ent ? b_org[k] : ws.org[k - base_ent]; }
+  __device__ const uint32_t* ebits(long long k) const {
+    return k < base_ent ? b_bits + (size_t)k * W : ws.bits + (size_t)(k - base_ent) * W;
+  }
+  __device__ uint32_t esum(long long k, int which) const {
+    return k < base_ent ? b_esum[(size_t)k * 2 + which] : ws.esum[(size_t)(k - base_ent) * 2 + which];
   }
 
   // ------------------------------------------------------------ bitmaps
@@ -327,13 +373,13 @@ class WarpWalker {
   // terminals, -1: none) tested against `fold`.
   __device__ void scatter(int col, const uint32_t* M, bool shift, int which, uint32_t fold) {
     const int lane = wl_lane();
-    const int b = ws.col_off[col], e = ws.col_off[col + 1];
-    for (int base = b; base < e; base += 32) {
-      int k = base + lane;
-      bool act = k < e && (which < 0 || (ws.esum[(size_t)k * 2 + which] & fold) != 0);
+    const long long b = cbeg(col), e = cend(col);
+    for (long long base = b; base < e; base += 32) {
+      long long k = base + lane;
+      bool act = k < e && (which < 0 || (esum(k, which) & fold) != 0);
       unsigned am = __ballot_sync(0xffffffffu, act);
       if (!am) continue;
-      int o2 = act ? ws.org[k] : -1;
+      int o2 = act ? eorg(k) : -1;
       uint32_t* dst = nullptr;
       if constexpr (SM) {
         bool need = act && slot_of[o2] < 0;
@@ -360,7 +406,7 @@ class WarpWalker {
       }
       bool ch = false;
       if (act) {
-        const uint32_t* src = ws.bits + (size_t)k * W;
+        const uint32_t* src = ebits(k);
         uint32_t carry = 0;
         for (int w = 0; w < W; ++w) {
           uint32_t v = M ? (src[w] & M[w]) : src[w];
@@ -389,6 +435,7 @@ class WarpWalker {
       status = 1;
       return -1;
     }
+    cur_col = ncols;
     return ncols;
   }
   __device__ void arrive(int src, const uint32_t* M, bool shift) {
@@ -396,7 +443,22 @@ class WarpWalker {
     arrive_inner(src, M, shift);
     PH_END(1, t_arr);
   }
+  __device__ void record_edge(int src, bool labelled) {
+    if (wl_lane() == 0) {
+      if (rec->n_edges >= rec->edge_cap) {
+        status = 1;
+      } else {
+        int e = rec->n_edges++;
+        rec->e_dst[e] = cur_col;
+        rec->e_src[e] = src;
+        for (int w = 0; w < 8; ++w) rec->e_lbl[(size_t)e * 8 + w] = labelled ? cur_lbl8[w] : 0u;
+      }
+    }
+    status = __shfl_sync(0xffffffffu, status, 0);
+    rec->n_edges = __shfl_sync(0xffffffffu, rec->n_edges, 0);
+  }
   __device__ void arrive_inner(int src, const uint32_t* M, bool shift) {
+    if (rec) record_edge(src, shift);
     if (shift)
       scatter(src, M, true, 1, label_fold);
     else
@@ -411,7 +473,32 @@ class WarpWalker {
     bm_set(sh.dirty, c);
   }
 
+  // Suffix mode (a check's nodes after its region): no predictions, and rows
+  // whose origin is a base-chart column are not closed here -- whether such
+  // an item leads to acceptance is read from the base chart's good masks at
+  // node res_node when the column is finished (found = 1); they are not kept.
+  bool suffix_mode = false;
+  int res_node = -1;
+  const uint32_t* good = nullptr;
+  int found = 0;
+  int region_start = -1;  // own start column (S' item has an own origin) or -1
+  int accept_node = -1;   // the base chart's accept node
+
+  // entry of base-chart column j with origin o, or -1
+  __device__ long long find_base(int j, int o) const {
+    long long lo = b_col_off[j], hi = b_col_off[j + 1];
+    for (long long base = lo; base < hi; base += 32) {
+      long long k = base + wl_lane();
+      bool hit = k < hi && b_org[k] == o;
+      unsigned m = __ballot_sync(0xffffffffu, hit);
+      if (m) return base + __ffs(m) - 1;
+    }
+    return -1;
+  }
+
+  bool cur_gap = false;
   __device__ void close_column(int c, bool gap) {
+    cur_gap = gap;
     const uint32_t* P = gap ? g.gap_pred : g.pred;
     for (long long it = 0;; ++it) {
       if (it > kWMaxSteps) {
@@ -419,6 +506,14 @@ class WarpWalker {
         return;
       }
       int o = bm_highest(sh.dirty, c + 1);
+      if (suffix_mode) {
+        if (o < 0) break;
+        if (o < base_cols) {  // resolved by the good masks at finish
+          if (wl_lane() == 0) sh.dirty[o >> 5] &= ~(1u << (o & 31));
+          __syncwarp();
+          continue;
+        }
+      }
       if (o < 0) {
         // predictions for origin c from the nonterminals waited on here
         bool any = false;
@@ -499,13 +594,25 @@ class WarpWalker {
     PH_END(7, t_fin);
   }
   __device__ void finish_inner(int c) {
-    long long E = ws.col_off[c];
+    const int oc = c - base_cols;  // own column index
+    long long E = ws.col_off[oc];
     int o = -1;
     while ((o = bm_next(sh.touched, o + 1, c + 1)) >= 0) {
       uint32_t* row = row_of(o);
       bool nz = false;
       for (int w = wl_lane(); w < W; w += 32) nz |= row[w] != 0;
       nz = __any_sync(0xffffffffu, nz);
+      if (nz && suffix_mode && o < base_cols) {
+        long long kf = find_base(res_node, o);
+        bool hit = false;
+        if (kf >= 0)
+          for (int w = wl_lane(); w < W; w += 32) hit |= (row[w] & good[(size_t)kf * W + w]) != 0;
+        if (__any_sync(0xffffffffu, hit)) found = 1;
+        nz = false;  // not kept
+      }
+      if (nz && suffix_mode && o == region_start && res_node == accept_node &&
+          ((row[g.accept_item >> 5] >> (g.accept_item & 31)) & 1u))
+        found = 1;
       if (nz) {
         if (E >= emax) {
           status = 1;
@@ -518,6 +625,12 @@ class WarpWalker {
           }
           uint32_t* dst = ws.bits + (size_t)E * W;
           for (int w = wl_lane(); w < W; w += 32) dst[w] = row[w];
+          if (rec) {  // completed nonterminals of the entry
+            for (int v = wl_lane(); v < VW; v += 32) sh.nt[v] = 0;
+            __syncwarp();
+            row_nts(row, g.complete, true, sh.nt);
+            for (int v = wl_lane(); v < VW; v += 32) rec->cnt[(size_t)E * VW + v] = sh.nt[v];
+          }
           ++E;
         }
       }
@@ -532,12 +645,15 @@ class WarpWalker {
       sh.vset[v] = 0;
       sh.vdone[v] = 0;
     }
-    if (wl_lane() == 0) ws.col_off[c + 1] = (int)E;
+    if (wl_lane() == 0) {
+      ws.col_off[oc + 1] = (int)E;
+      if (rec) rec->col_gap[c] = cur_gap ? 1 : 0;
+    }
     __syncwarp();
     nent = E;
     ncols = c + 1;
   }
-  __device__ bool column_empty(int c) { return ws.col_off[c + 1] == ws.col_off[c]; }
+  __device__ bool column_empty(int c) { return cend(c) == cbeg(c); }
 
   // abandon the open column: zero its rows
   __device__ void cleanup() {
@@ -560,16 +676,18 @@ class WarpWalker {
 
   __device__ bool accepts(int c, int start) {
     bool f = false;
-    for (int k = ws.col_off[c] + wl_lane(); k < ws.col_off[c + 1]; k += 32)
-      if (ws.org[k] == start && ((ws.bits[(size_t)k * W + (g.accept_item >> 5)] >> (g.accept_item & 31)) & 1u))
-        f = true;
+    for (long long k = cbeg(c) + wl_lane(); k < cend(c); k += 32)
+      if (eorg(k) == start && ((ebits(k)[g.accept_item >> 5] >> (g.accept_item & 31)) & 1u)) f = true;
     return __any_sync(0xffffffffu, f);
   }
 
   // ------------------------------------------------------------ labels
   __device__ void label_set(const uint32_t* lbl8) {
     label_fold = 0;
-    for (int lw = 0; lw < 8; ++lw) label_fold |= lbl8[lw];
+    for (int lw = 0; lw < 8; ++lw) {
+      label_fold |= lbl8[lw];
+      cur_lbl8[lw] = lbl8[lw];
+    }
     for (int w = wl_lane(); w < W; w += 32) {
       uint32_t acc = 0;
       for (int lw = 0; lw < 8; ++lw) {
@@ -587,6 +705,7 @@ class WarpWalker {
   }
   __device__ void label_one(int a) {
     label_fold = 1u << (a & 31);
+    for (int lw = 0; lw < 8; ++lw) cur_lbl8[lw] = (lw == (a >> 5)) ? (1u << (a & 31)) : 0u;
     for (int w = wl_lane(); w < W; w += 32) sh.lbl[w] = g.exp_term[(size_t)a * W + w];
     __syncwarp();
   }
@@ -737,13 +856,13 @@ class WarpWalker {
 
   // x (+) {(sp, st)}; returns 1 valid, 0 invalid, -1 overflow, -2 bad input
   __device__ int run(const int32_t* x, int n, int sp, int st) {
-    ncols = 0;
+    ncols = base_cols;
     nent = 0;
     status = 0;
     nf = 0;
     if (wl_lane() == 0) ws.col_off[0] = 0;
     __syncwarp();
-    if (sp < 0 || sp >= n || x[sp] >= 0 || st < 0 || st >= vocab) return -2;
+    if (sp >= 0 && (sp >= n || x[sp] >= 0 || st < 0 || st >= vocab)) return -2;
     int r = run_inner(x, n, sp, st);
     if (r < 0 || status) {
       cleanup();
@@ -752,39 +871,94 @@ class WarpWalker {
     return r;
   }
 
+  // a gap node after the span in the frontier: a pending lexeme some byte
+  // can extend stays open (epsilon), one no byte can extend emits its terminal
+  __device__ int gap_from_frontier() {
+    int c = open_column();
+    if (c < 0) return -1;
+    for (int f = 0; f < nf; ++f) {
+      int q = ws.f_q[f];
+      int a = g.dfa_accept[q];
+      if (q == 0 || g.dfa_ext[q] || (a >= 0 && g.skip[a])) {
+        arrive(ws.f_c[f], nullptr, false);
+      } else if (a >= 0) {
+        label_one(a);
+        arrive(ws.f_c[f], sh.lbl, true);
+      }
+    }
+    return c;
+  }
+  // the END node: the pending lexeme is flushed
+  __device__ int end_from_frontier() {
+    int c = open_column();
+    if (c < 0) return -1;
+    for (int f = 0; f < nf; ++f) {
+      int q = ws.f_q[f];
+      int a = g.dfa_accept[q];
+      if (q == 0 || (a >= 0 && g.skip[a])) {
+        arrive(ws.f_c[f], nullptr, false);
+      } else if (a >= 0) {
+        label_one(a);
+        arrive(ws.f_c[f], sh.lbl, true);
+      }
+    }
+    return c;
+  }
+  // frontier of a span that starts at column src: q0 at the sequence start,
+  // every lexer state after a gap
+  __device__ void frontier_from(int src, bool at_begin) {
+    if (at_begin) {
+      if (wl_lane() == 0) {
+        ws.f_q[0] = 0;
+        ws.f_c[0] = src;
+      }
+      nf = 1;
+    } else {
+      for (int q = wl_lane(); q < g.Q; q += 32) {
+        ws.f_q[q] = q;
+        ws.f_c[q] = src;
+      }
+      nf = g.Q;
+    }
+    __syncwarp();
+  }
+  __device__ void rec_range(int32_t* arr, int lo, int hi, int v) {
+    for (int p = lo + (int)wl_lane(); p < hi; p += 32) arr[p] = v;
+    __syncwarp();
+  }
+
   __device__ int run_inner(const int32_t* x, int n, int sp, int stok) {
     int i = 0;
     bool first = true;
     int prev_gap = -1;
+    int span_lo = -1, span_hi = -1;  // the last span, for post_col
     while (i < n) {
       int t0 = token_at(x, sp, stok, i);
       int j = i;
       if (t0 < 0) {
         while (j < n && token_at(x, sp, stok, j) < 0) ++j;
-        int c = open_column();
-        if (c < 0) return -1;
+        int c;
         if (first) {
+          c = open_column();
+          if (c < 0) return -1;
           start_col = c;
           seed(c);
         } else {
-          for (int f = 0; f < nf; ++f) {
-            int q = ws.f_q[f];
-            int a = g.dfa_accept[q];
-            if (q == 0 || g.dfa_ext[q] || (a >= 0 && g.skip[a])) {
-              arrive(ws.f_c[f], nullptr, false);
-            } else if (a >= 0) {
-              label_one(a);
-              arrive(ws.f_c[f], sh.lbl, true);
-            }
-          }
+          c = gap_from_frontier();
+          if (c < 0) return -1;
         }
         close_column(c, true);
         finish_column(c);
         if (status) return -1;
+        if (rec) {
+          rec_range(rec->gap_col, i, j, c);
+          if (span_lo >= 0) rec_range(rec->post_col, span_lo, span_hi, c);
+        }
         prev_gap = c;
         if (column_empty(c)) return 0;
       } else {
         while (j < n && token_at(x, sp, stok, j) >= 0) ++j;
+        int src;
         if (first) {
           int c = open_column();
           if (c < 0) return -1;
@@ -793,20 +967,14 @@ class WarpWalker {
           close_column(c, false);
           finish_column(c);
           if (status) return -1;
-          if (wl_lane() == 0) {
-            ws.f_q[0] = 0;
-            ws.f_c[0] = c;
-          }
-          __syncwarp();
-          nf = 1;
+          src = c;
         } else {
-          for (int q = wl_lane(); q < g.Q; q += 32) {
-            ws.f_q[q] = q;
-            ws.f_c[q] = prev_gap;
-          }
-          __syncwarp();
-          nf = g.Q;
+          src = prev_gap;
         }
+        frontier_from(src, first);
+        if (rec) rec_range(rec->pre_col, i, j, src);
+        span_lo = i;
+        span_hi = j;
         for (int p = i; p < j && nf > 0; ++p) {
           int tok = token_at(x, sp, stok, p);
           if (tok < 0 || tok >= vocab) return -2;
@@ -814,27 +982,22 @@ class WarpWalker {
         }
         if (nf == 0) return 0;
         if (j == n) {  // END: flush the pending lexeme
-          int c = open_column();
+          int c = end_from_frontier();
           if (c < 0) return -1;
-          for (int f = 0; f < nf; ++f) {
-            int q = ws.f_q[f];
-            int a = g.dfa_accept[q];
-            if (q == 0 || (a >= 0 && g.skip[a])) {
-              arrive(ws.f_c[f], nullptr, false);
-            } else if (a >= 0) {
-              label_one(a);
-              arrive(ws.f_c[f], sh.lbl, true);
-            }
-          }
           close_column(c, false);
           finish_column(c);
           if (status) return -1;
+          if (rec) {
+            rec_range(rec->post_col, i, j, c);
+            if (wl_lane() == 0) rec->meta[3] = c;
+          }
           return accepts(c, start_col) ? 1 : 0;
         }
       }
       first = false;
       i = j;
     }
+    if (rec && wl_lane() == 0) rec->meta[3] = prev_gap;
     return accepts(prev_gap, start_col) ? 1 : 0;
   }
 };

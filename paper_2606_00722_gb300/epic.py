@@ -17,7 +17,7 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = [os.path.join(_HERE, 'csrc', f) for f in ('epic.cu', 'grammar.cpp')]
 _DEPS = _SRC + [os.path.join(_HERE, 'csrc', f) for f in
-                ('grammar.h', 'device.cuh', 'walk.cuh', 'cover.cuh', 'skeleton.cuh', 'warpwalk.cuh')] + \
+                ('grammar.h', 'device.cuh', 'walk.cuh', 'cover.cuh', 'skeleton.cuh', 'warpwalk.cuh', 'region.cuh')] + \
     [os.path.join(_HERE, '..', 'include', 'epic.h')]
 LIB_PATH = os.path.join(_HERE, '_build', 'libepic.so')
 NVCC_FLAGS = ['-gencode', 'arch=compute_103a,code=sm_103a', '-lineinfo', '-O3', '-std=c++17',
