@@ -801,7 +801,7 @@ epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const in
     }
   }
   // 2. good masks
-  k_good<<<(B + kWarpsPerCta - 1) / kWarpsPerCta, 32 * kWarpsPerCta, 0, st>>>(dg, B, sp);
+  k_good<<<B, 32 * kGoodWarps, 0, st>>>(dg, B, sp);
   // 3. checks
   cudaMemsetAsync(t->d_counter, 0, 8, st);
   size_t per = smem_per_warp(wp.nmax, rmax, dg.W, dg.VW);
@@ -1074,8 +1074,11 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
   if (total == 0) return EPIC_OK;
   if (!d_x || !d_pos || !d_cand || !d_valid || n == 0) return EPIC_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)cuda_stream;
-  // wide item sets (large grammars): checks by region over a per-sequence chart
-  bool region = g->dg.W > 32;
+  // Checks by region over a per-sequence chart when the item sets are wide
+  // (whole-graph walks of large grammars are far too long) or when there are
+  // more checks than resident walks: the chart of x is then built once per
+  // sequence instead of once per check.
+  bool region = g->dg.W > 32 || total > (long long)sm_count() * 2 * kWarpsPerCta;
   if (const char* e = getenv("EPIC_REGION")) region = atoi(e) != 0;
   if (region) return validate_region(g, t, d_x, B, n, d_pos, k, d_cand, K, d_valid, st);
   epic_status s = ensure_wworkspace(t, total, n, st);

@@ -37,6 +37,9 @@ struct SeqArena {
   int32_t* succ_off;   // [nmax + 1] columns holding origin u, ascending
   int32_t* succ_idx;   // [emax]
   uint32_t* expn;      // [nmax][W] scratch of the good pass
+  int32_t* eidx;       // [nmax (nmax + 1) / 2] entry of (column j, origin o <= j), -1: none
+  uint8_t* gnz;        // [emax] the entry has a good item
+  int32_t* cursor;     // [2 (nmax + 1)] scratch of the good pass
 };
 
 struct SeqPack {
@@ -52,7 +55,7 @@ struct SeqPack {
            + r(nm) + 2 * r((size_t)edge_cap * 4) + r((size_t)edge_cap * 32) + 3 * r((size_t)n * 4) +
            r((size_t)emax * VW * 4) + r(32)                                                 // SeqRec
            + r((size_t)emax * W * 4) + r(nm * 4) + 3 * r((nm + 1) * 4) + r((size_t)edge_cap * 4) +
-           r((size_t)emax * 4) + r(nm * W * 4);
+           r((size_t)emax * 4) + r(nm * W * 4) + r(nm * (nm + 1) / 2 * 4) + r((size_t)emax) + r(2 * (nm + 1) * 4);
   }
   __device__ SeqArena carve(long long b) const {
     SeqArena a;
@@ -97,6 +100,9 @@ struct SeqPack {
     a.out_idx = (int32_t*)take((size_t)edge_cap * 4);
     a.succ_idx = (int32_t*)take((size_t)emax * 4);
     a.expn = (uint32_t*)take(nm * W * 4);
+    a.eidx = (int32_t*)take(nm * (nm + 1) / 2 * 4);
+    a.gnz = (uint8_t*)take((size_t)emax);
+    a.cursor = (int32_t*)take(2 * (nm + 1) * 4);
     return a;
   }
 };
@@ -166,205 +172,200 @@ __device__ __forceinline__ uint32_t shr1_word(const uint32_t* src, int w, int W)
   return v;
 }
 
-__global__ void __launch_bounds__(32 * kWarpsPerCta) k_good(DevGrammar g, int B, SeqPack sp) {
-  int warp = threadIdx.x >> 5;
-  long long b = (long long)blockIdx.x * (blockDim.x >> 5) + warp;
+constexpr int kGoodWarps = 32;  // one CTA per sequence
+
+// Good items of a sequence's forward chart, columns from last to first.
+// Item i of entry (j, o) is good when it is present and
+//  - it is the accepting item at the accept node with the start origin;
+//  - an out-edge j -> j2 scans a terminal it expects (or is epsilon) and the
+//    advanced item of (j2, o) is good;
+//  - it waits on a nonterminal that completes from origin j at column j2
+//    (j2 = j: a nullable one) and the advanced item of (j2, o) is good;
+//  - j is a gap and the item advanced over any symbol is good;
+//  - it is complete with left side B, and some item of column o, origin o2,
+//    waiting on B has its advanced item good at (j, o2).
+// The first three read later columns only (final); the last two read this
+// column: its entries iterate to the least fixpoint together.
+__global__ void __launch_bounds__(32 * kGoodWarps) k_good(DevGrammar g, int B, SeqPack sp) {
+  const long long b = blockIdx.x;
   if (b >= B) return;
-  const int lane = threadIdx.x & 31;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nthr = blockDim.x;
   const int W = g.W, VW = g.VW;
   SeqArena a = sp.carve(b);
-  const int32_t* meta = a.rec.meta;
+  int32_t* meta = a.rec.meta;
   if (meta[M_STATUS] != 1) return;
   const int N = meta[M_NCOLS], NE = meta[M_NEDGES];
   const int32_t* col = a.ws.col_off;
-  const long long E = col[N];
+  const int32_t* org = a.ws.org;
   const int start = meta[M_START], accept = meta[M_ACCEPT];
-  // in-edge offsets (edges are stored in target order), out-edge CSR
-  for (int j = lane; j <= N; j += 32) {
+  __shared__ int s_flag;
+  __shared__ uint32_t s_nt[kGoodWarps][kWMaxVW];
+  int32_t* cur_o = a.cursor;          // [N + 1]
+  int32_t* cur_s = a.cursor + N + 1;  // [N + 1]
+  // edges by source and entries by origin (CSR), entry index by (column, origin)
+  for (int j = tid; j <= N; j += nthr) {
     a.in_off[j] = 0;
     a.out_off[j] = 0;
     a.succ_off[j] = 0;
   }
-  __syncwarp();
-  for (int e = lane; e < NE; e += 32) {
+  for (int u = tid; u < N; u += nthr) a.last_col[u] = -1;
+  const size_t ntri = (size_t)N * (N + 1) / 2;
+  for (size_t q = tid; q < ntri; q += nthr) a.eidx[q] = -1;
+  __syncthreads();
+  for (int e = tid; e < NE; e += nthr) {
     atomicAdd(&a.in_off[a.rec.e_dst[e] + 1], 1);
     atomicAdd(&a.out_off[a.rec.e_src[e] + 1], 1);
   }
-  for (long long k = lane; k < E; k += 32) atomicAdd(&a.succ_off[a.ws.org[k] + 1], 1);
-  __syncwarp();
-  if (lane == 0)
+  for (int j = warp; j < N; j += kGoodWarps)
+    for (long long k = col[j] + lane; k < col[j + 1]; k += 32) {
+      const int o = org[k];
+      a.eidx[tri_index(j, o)] = (int32_t)k;
+      a.gnz[k] = 0;
+      atomicAdd(&a.succ_off[o + 1], 1);
+      atomicMax(&a.last_col[o], j);
+    }
+  __syncthreads();
+  if (tid == 0)
     for (int j = 0; j < N; ++j) {
       a.in_off[j + 1] += a.in_off[j];
       a.out_off[j + 1] += a.out_off[j];
       a.succ_off[j + 1] += a.succ_off[j];
     }
-  __syncwarp();
-  int32_t* cur = a.last_col;  // cursor, reused below as last_col
-  for (int j = lane; j < N; j += 32) cur[j] = a.out_off[j];
-  __syncwarp();
-  for (int e = lane; e < NE; e += 32) a.out_idx[atomicAdd(&cur[a.rec.e_src[e]], 1)] = e;
-  __syncwarp();
-  for (int j = lane; j < N; j += 32) cur[j] = a.succ_off[j];
-  __syncwarp();
-  for (int c = 0; c < N; ++c)  // column by column: each list ascends
-    for (long long k = col[c] + lane; k < col[c + 1]; k += 32) a.succ_idx[atomicAdd(&cur[a.ws.org[k]], 1)] = c;
-  __syncwarp();
-  for (int u = lane; u < N; u += 32)
-    a.last_col[u] = a.succ_off[u + 1] > a.succ_off[u] ? a.succ_idx[a.succ_off[u + 1] - 1] : -1;
-  __syncwarp();
-  auto find = [&](int j, int o) -> long long {
-    long long lo = col[j], hi = col[j + 1];
-    for (long long base = lo; base < hi; base += 32) {
-      long long k = base + lane;
-      bool hit = k < hi && a.ws.org[k] == o;
-      unsigned m = __ballot_sync(0xffffffffu, hit);
-      if (m) return base + __ffs(m) - 1;
-    }
-    return -1;
-  };
-  constexpr int KW = kWMaxW / 32;
-  const int nw = (W + 31) >> 5;
-  __shared__ uint32_t s_nt[kWarpsPerCta][kWMaxVW];
-  uint32_t* bset = s_nt[warp];
+  __syncthreads();
+  for (int j = tid; j < N; j += nthr) {
+    cur_o[j] = a.out_off[j];
+    cur_s[j] = a.succ_off[j];
+  }
+  __syncthreads();
+  for (int e = tid; e < NE; e += nthr) a.out_idx[atomicAdd(&cur_o[a.rec.e_src[e]], 1)] = e;
+  for (int j = warp; j < N; j += kGoodWarps)
+    for (long long k = col[j] + lane; k < col[j + 1]; k += 32) a.succ_idx[atomicAdd(&cur_s[org[k]], 1)] = j;
+  __syncthreads();
+
+  uint32_t* G = a.good;
   for (int j = N - 1; j >= 0; --j) {
-    const bool gap = a.rec.col_gap[j] != 0;
-    // EXPN of what completes from origin j at each later column j2
     const int s0 = a.succ_off[j], s1 = a.succ_off[j + 1];
-    for (int si = s0; si < s1; ++si) {
-      int j2 = a.succ_idx[si];
-      long long kc = find(j2, j);
+    const bool gap = a.rec.col_gap[j] != 0;
+    const long long k0 = col[j], k1 = col[j + 1];
+    if (k0 == k1) continue;
+    // EXPN of what completes from origin j at each column j2 (j2 = j included)
+    int self_si = -1;
+    for (int si = s0; si < s1; ++si)
+      if (a.succ_idx[si] == j) self_si = si - s0;
+    for (int si = s0 + warp; si < s1; si += kGoodWarps) {
+      const int j2 = a.succ_idx[si];
+      const uint32_t* cn = a.rec.cnt + (size_t)a.eidx[tri_index(j2, j)] * VW;
+      expn_of_set(g, cn, a.expn + (size_t)(si - s0) * W);
+    }
+    __syncthreads();
+    // from the later columns: scans along the out-edges, nested constituents
+    for (long long k = k0 + warp; k < k1; k += kGoodWarps) {
+      const int o = org[k];
+      const uint32_t* bits = a.ws.bits + (size_t)k * W;
+      uint32_t* Gk = G + (size_t)k * W;
+      bool nz = false;
       for (int w = lane; w < W; w += 32) {
         uint32_t acc = 0;
-        for (int v = 0; v < VW; ++v) {
-          uint32_t m = a.rec.cnt[(size_t)kc * VW + v];
-          while (m) {
-            int bb = __ffs(m) - 1;
-            m &= m - 1;
-            acc |= g.exp_nt[(size_t)((v << 5) + bb) * W + w];
-          }
-        }
-        a.expn[(size_t)(si - s0) * W + w] = acc;
-      }
-    }
-    __syncwarp();
-    for (long long k = col[j]; k < col[j + 1]; ++k) {
-      const int o = a.ws.org[k];
-      const uint32_t* bits = a.ws.bits + (size_t)k * W;
-      uint32_t* G = a.good + (size_t)k * W;
-      for (int w = lane; w < W; w += 32) G[w] = 0;
-      __syncwarp();
-      if (j == accept && o == start && lane == 0)
-        G[g.accept_item >> 5] = bits[g.accept_item >> 5] & (1u << (g.accept_item & 31));
-      __syncwarp();
-      // each round that changes the row adds an item: W * 32 + 1 rounds reach the fixpoint
-      for (int round = 0; round <= W * 32; ++round) {
-        bool ch = false;
-        uint32_t acc[KW];
-#pragma unroll
-        for (int i = 0; i < KW; ++i) acc[i] = 0;
-        // (ii) scans and epsilon moves along the out-edges
+        if (j == accept && o == start && w == (g.accept_item >> 5)) acc |= 1u << (g.accept_item & 31);
         for (int ei = a.out_off[j]; ei < a.out_off[j + 1]; ++ei) {
-          int e = a.out_idx[ei];
-          int j2 = a.rec.e_dst[e];
-          long long k2 = find(j2, o);
-          if (k2 < 0) continue;
-          const uint32_t* G2 = a.good + (size_t)k2 * W;
+          const int e = a.out_idx[ei];
+          const int k2 = a.eidx[tri_index(a.rec.e_dst[e], o)];
+          if (k2 < 0 || !a.gnz[k2]) continue;
+          const uint32_t* G2 = G + (size_t)k2 * W;
           const uint32_t* L = a.rec.e_lbl + (size_t)e * 8;
+          uint32_t m = 0;
           bool eps = true;
-          for (int lw = 0; lw < 8; ++lw) eps &= L[lw] == 0;
-#pragma unroll
-          for (int i = 0; i < KW; ++i) {
-            int w = lane + 32 * i;
-            if (i < nw && w < W) {
-              uint32_t m = 0xffffffffu;
-              if (!eps) {
-                m = 0;
-                for (int lw = 0; lw < 8; ++lw) {
-                  uint32_t lm = L[lw];
-                  while (lm) {
-                    int bb = __ffs(lm) - 1;
-                    lm &= lm - 1;
-                    int t = (lw << 5) + bb;
-                    if (t < g.T) m |= g.exp_term[(size_t)t * W + w];
-                  }
-                }
-                acc[i] |= bits[w] & m & shr1_word(G2, w, W);
-              } else {
-                acc[i] |= bits[w] & G2[w];
+          for (int lw = 0; lw < 8; ++lw) {
+            uint32_t lm = L[lw];
+            eps &= lm == 0;
+            while (lm) {
+              const int bb = __ffs(lm) - 1;
+              lm &= lm - 1;
+              const int t = (lw << 5) + bb;
+              if (t < g.T) m |= g.exp_term[(size_t)t * W + w];
+            }
+          }
+          acc |= eps ? G2[w] : (m & shr1_word(G2, w, W));
+        }
+        for (int si = s0; si < s1; ++si) {
+          if (si - s0 == self_si) continue;
+          const int k3 = a.eidx[tri_index(a.succ_idx[si], o)];
+          if (k3 < 0 || !a.gnz[k3]) continue;
+          acc |= a.expn[(size_t)(si - s0) * W + w] & shr1_word(G + (size_t)k3 * W, w, W);
+        }
+        const uint32_t v = bits[w] & acc;
+        Gk[w] = v;
+        nz |= v != 0;
+      }
+      nz = __any_sync(0xffffffffu, nz);
+      if (lane == 0) a.gnz[k] = nz ? 1 : 0;
+    }
+    __syncthreads();
+    // completions within the column and the self rules, to the fixpoint
+    for (int pass = 0;; ++pass) {
+      if (pass > (1 << 20)) {  // cannot happen before the fixpoint; never silently wrong
+        if (tid == 0) meta[M_STATUS] = -1;
+        return;
+      }
+      if (tid == 0) s_flag = 0;
+      __syncthreads();
+      bool changed = false;
+      uint32_t* bset = s_nt[warp];
+      for (long long k = k0 + warp; k < k1; k += kGoodWarps) {
+        const int o = org[k];
+        const uint32_t* bits = a.ws.bits + (size_t)k * W;
+        uint32_t* Gk = G + (size_t)k * W;
+        // each round that changes the entry adds an item
+        for (int round = 0; round <= W * 32; ++round) {
+          for (int v = lane; v < VW; v += 32) bset[v] = 0;
+          __syncwarp();
+          for (long long kp = col[o]; kp < col[o + 1]; ++kp) {
+            const int o2 = org[kp];
+            const long long kk = (o2 == o) ? k : a.eidx[tri_index(j, o2)];
+            if (kk < 0 || (kk != k && !a.gnz[kk])) continue;
+            const uint32_t* P = a.ws.bits + (size_t)kp * W;
+            const uint32_t* GK = G + (size_t)kk * W;
+            for (int w = lane; w < W; w += 32) {
+              uint32_t m = P[w] & g.any_nt[w] & shr1_word(GK, w, W);
+              while (m) {
+                const int bb = __ffs(m) - 1;
+                m &= m - 1;
+                const int Bn = g.item_next[(w << 5) + bb] - g.T;
+                atomicOr(&bset[Bn >> 5], 1u << (Bn & 31));
               }
             }
           }
-        }
-        // (iv) nested constituents completing from j at j2 (j2 = j: this row)
-        for (int si = s0; si < s1; ++si) {
-          int j2 = a.succ_idx[si];
-          long long k3 = (j2 == j) ? k : find(j2, o);
-          if (k3 < 0) continue;
-          const uint32_t* G3 = a.good + (size_t)k3 * W;
-#pragma unroll
-          for (int i = 0; i < KW; ++i) {
-            int w = lane + 32 * i;
-            if (i < nw && w < W) acc[i] |= bits[w] & a.expn[(size_t)(si - s0) * W + w] & shr1_word(G3, w, W);
-          }
-        }
-        // inside a gap every item advances over any symbol
-        if (gap) {
-#pragma unroll
-          for (int i = 0; i < KW; ++i) {
-            int w = lane + 32 * i;
-            if (i < nw && w < W) acc[i] |= bits[w] & g.next_any[w] & shr1_word(G, w, W);
-          }
-        }
-        // (v) completion: the items of column o waiting on the completed
-        // nonterminal advance to good items of this node
-        for (int v = lane; v < VW; v += 32) bset[v] = 0;
-        __syncwarp();
-        for (long long kp = col[o]; kp < col[o + 1]; ++kp) {
-          int o2 = a.ws.org[kp];
-          long long kk = (o2 == o) ? k : find(j, o2);
-          if (kk < 0) continue;
-          const uint32_t* P = a.ws.bits + (size_t)kp * W;
-          const uint32_t* GK = a.good + (size_t)kk * W;
+          __syncwarp();
+          bool ch = false;
           for (int w = lane; w < W; w += 32) {
-            uint32_t m = P[w] & g.any_nt[w] & shr1_word(GK, w, W);
-            while (m) {
-              int bb = __ffs(m) - 1;
-              m &= m - 1;
-              int Bn = g.item_next[(w << 5) + bb] - g.T;
-              atomicOr(&bset[Bn >> 5], 1u << (Bn & 31));
-            }
-          }
-        }
-        __syncwarp();
-#pragma unroll
-        for (int i = 0; i < KW; ++i) {
-          int w = lane + 32 * i;
-          if (i < nw && w < W) {
-            uint32_t m = bits[w] & g.complete[w];
             uint32_t add = 0;
+            uint32_t m = bits[w] & g.complete[w];
             while (m) {
-              int bb = __ffs(m) - 1;
+              const int bb = __ffs(m) - 1;
               m &= m - 1;
-              int L2 = g.item_lhs[(w << 5) + bb];
+              const int L2 = g.item_lhs[(w << 5) + bb];
               if ((bset[L2 >> 5] >> (L2 & 31)) & 1u) add |= 1u << bb;
             }
-            acc[i] |= add;
-          }
-        }
-#pragma unroll
-        for (int i = 0; i < KW; ++i) {
-          int w = lane + 32 * i;
-          if (i < nw && w < W) {
-            uint32_t old = G[w];
-            if ((old | acc[i]) != old) {
-              G[w] = old | acc[i];
+            const uint32_t s = shr1_word(Gk, w, W);
+            if (gap) add |= g.next_any[w] & s;
+            if (self_si >= 0) add |= a.expn[(size_t)self_si * W + w] & s;
+            add &= bits[w];
+            const uint32_t old = Gk[w];
+            if ((old | add) != old) {
+              Gk[w] = old | add;
               ch = true;
             }
           }
+          if (!__any_sync(0xffffffffu, ch)) break;
+          changed = true;
+          if (lane == 0) a.gnz[k] = 1;
         }
-        __syncwarp();
-        if (!__any_sync(0xffffffffu, ch)) break;
       }
+      if (changed && lane == 0) s_flag = 1;
+      __syncthreads();
+      const int more = s_flag;
+      __syncthreads();
+      if (!more) break;
     }
   }
 }
@@ -391,6 +392,7 @@ struct RegionCheck {
     w.b_bits = a.ws.bits;
     w.b_esum = a.ws.esum;
     w.good = a.good;
+    w.b_eidx = a.eidx;
     w.accept_node = meta[M_ACCEPT];
     w.ncols = NF;
     w.nent = 0;
@@ -517,18 +519,7 @@ struct RegionCheck {
         uint32_t fold = 0;
         for (int v = 0; v < w.VW; ++v) fold |= w.sh.nt[v];
         if (!fold) continue;
-        for (int ww = lane; ww < w.W; ww += 32) {
-          uint32_t acc = 0;
-          for (int v = 0; v < w.VW; ++v) {
-            uint32_t m = w.sh.nt[v];
-            while (m) {
-              int bb = __ffs(m) - 1;
-              m &= m - 1;
-              acc |= w.g.exp_nt[(size_t)((v << 5) + bb) * w.W + ww];
-            }
-          }
-          w.sh.expn[ww] = acc;
-        }
+        expn_of_set(w.g, w.sh.nt, w.sh.expn);
         __syncwarp();
         w.scatter(u, w.sh.expn, true, 0, fold);
         if (w.status) return -1;

@@ -22,6 +22,9 @@ constexpr int kWMaxVW = 32;
 constexpr int kWMaxQ = 1024;
 constexpr long long kWMaxSteps = 1ll << 24;  // closure iterations per column
 
+// index of (column j, origin o <= j) in a lower-triangular table
+__host__ __device__ __forceinline__ size_t tri_index(int j, int o) { return (size_t)j * (j + 1) / 2 + o; }
+
 struct WWs {  // per-warp global workspace
   uint32_t* stage;   // [nmax][W]
   uint32_t* bdone;   // [nmax][VW]
@@ -68,6 +71,42 @@ struct WSh {  // per-warp shared memory
 
 __device__ __forceinline__ uint32_t wl_lane() { return threadIdx.x & 31; }
 
+// Warp: out[w] = items waiting on a member of the nonterminal set nts
+// (VW words, readable by every lane), for the lane's words w.  A small set
+// ORs its EXP_NT rows; a large one tests each item's next symbol instead
+// (both give exactly the items whose next symbol is in the set).
+__device__ __forceinline__ void expn_of_set(const DevGrammar& g, const uint32_t* nts, uint32_t* out) {
+  const int W = g.W, VW = g.VW;
+  int cnt = 0;
+  for (int v = 0; v < VW; ++v) cnt += __popc(nts[v]);
+  if (cnt <= 24) {
+    for (int w = wl_lane(); w < W; w += 32) {
+      uint32_t acc = 0;
+      for (int v = 0; v < VW; ++v) {
+        uint32_t m = nts[v];
+        while (m) {
+          const int b = __ffs(m) - 1;
+          m &= m - 1;
+          acc |= g.exp_nt[(size_t)((v << 5) + b) * W + w];
+        }
+      }
+      out[w] = acc;
+    }
+  } else {
+    for (int w = wl_lane(); w < W; w += 32) {
+      uint32_t acc = 0;
+      const int i0 = w << 5;
+#pragma unroll 8
+      for (int b = 0; b < 32; ++b) {
+        const int i = i0 + b;
+        const int s = i < g.D ? g.item_next[i] - g.T : -1;
+        if (s >= 0 && ((nts[s >> 5] >> (s & 31)) & 1u)) acc |= 1u << b;
+      }
+      out[w] = acc;
+    }
+  }
+}
+
 #ifdef EPIC_PHASE_TIMERS
 __device__ unsigned long long g_phase[16];
 #define PH_BEGIN(v) long long v = clock64()
@@ -81,12 +120,11 @@ __device__ unsigned long long g_phase[16];
 #endif
 
 // SM = true keeps the rows of the column under construction in shared memory
-// (slot-mapped, rmax rows) and handles item sets of at most 32 words (one
-// word per lane); SM = false keeps them in the per-warp global stage and
-// handles up to kWMaxW words.
-template <bool SM>
+// (slot-mapped, rmax rows); SM = false keeps them in the per-warp global
+// stage.  KWv item words per lane: rows of up to 32 KWv words.
+template <bool SM, int KWv = (SM ? 1 : kWMaxW / 32)>
 class WarpWalker {
-  static constexpr int KW = SM ? 1 : kWMaxW / 32;  // item words per lane
+  static constexpr int KW = KWv;  // item words per lane
 
  public:
   // shared-memory staging (SM): rows [rmax][W], completed-NT sets [rmax][VW],
@@ -374,6 +412,71 @@ class WarpWalker {
   __device__ void scatter(int col, const uint32_t* M, bool shift, int which, uint32_t fold) {
     const int lane = wl_lane();
     const long long b = cbeg(col), e = cend(col);
+    if (W > 16) {  // wide rows: the lanes share each entry's words
+      for (long long base = b; base < e; base += 32) {
+        const long long k = base + lane;
+        const bool act = k < e && (which < 0 || (esum(k, which) & fold) != 0);
+        unsigned am = __ballot_sync(0xffffffffu, act);
+        const int my_org = act ? eorg(k) : -1;
+        while (am) {  // up to four entries at a time: their loads overlap
+          int ls[4];
+          int nl = 0;
+          while (am && nl < 4) {
+            ls[nl++] = __ffs(am) - 1;
+            am &= am - 1;
+          }
+          const uint32_t* src[4];
+          uint32_t* dst[4];
+          int o2[4];
+          uint32_t carry[4];
+          bool ch[4];
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const int l = i < nl ? ls[i] : ls[0];
+            o2[i] = __shfl_sync(0xffffffffu, my_org, l);
+            src[i] = ebits(base + l);
+            dst[i] = i < nl ? row_of(o2[i]) : nullptr;
+            carry[i] = 0;
+            ch[i] = false;
+          }
+          if (status) return;  // no shared-memory slot left
+          for (int w0 = 0; w0 < W; w0 += 32) {
+            const int w = w0 + lane;
+            const uint32_t m = (M && w < W) ? M[w] : 0xffffffffu;
+            uint32_t v[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) v[i] = (i < nl && w < W) ? (src[i][w] & m) : 0u;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+              uint32_t add = v[i];
+              if (shift) {
+                uint32_t prev = __shfl_up_sync(0xffffffffu, v[i], 1);
+                if (lane == 0) prev = carry[i];
+                add = (v[i] << 1) | (prev >> 31);
+                carry[i] = __shfl_sync(0xffffffffu, v[i], 31);
+              }
+              if (i < nl && w < W && add) {
+                const uint32_t old = dst[i][w];
+                if ((old | add) != old) {
+                  dst[i][w] = old | add;
+                  ch[i] = true;
+                }
+              }
+            }
+          }
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            const bool any = __any_sync(0xffffffffu, ch[i]);
+            if (i < nl && any && lane == 0) {
+              sh.touched[o2[i] >> 5] |= 1u << (o2[i] & 31);
+              sh.dirty[o2[i] >> 5] |= 1u << (o2[i] & 31);
+            }
+          }
+          __syncwarp();
+        }
+      }
+      return;
+    }
     for (long long base = b; base < e; base += 32) {
       long long k = base + lane;
       bool act = k < e && (which < 0 || (esum(k, which) & fold) != 0);
@@ -485,16 +588,8 @@ class WarpWalker {
   int accept_node = -1;   // the base chart's accept node
 
   // entry of base-chart column j with origin o, or -1
-  __device__ long long find_base(int j, int o) const {
-    long long lo = b_col_off[j], hi = b_col_off[j + 1];
-    for (long long base = lo; base < hi; base += 32) {
-      long long k = base + wl_lane();
-      bool hit = k < hi && b_org[k] == o;
-      unsigned m = __ballot_sync(0xffffffffu, hit);
-      if (m) return base + __ffs(m) - 1;
-    }
-    return -1;
-  }
+  const int32_t* b_eidx = nullptr;  // [(j (j + 1) / 2) + o] for o <= j
+  __device__ long long find_base(int j, int o) const { return o > j ? -1 : (long long)b_eidx[tri_index(j, o)]; }
 
   bool cur_gap = false;
   __device__ void close_column(int c, bool gap) {
@@ -565,18 +660,7 @@ class WarpWalker {
       if (!__any_sync(0xffffffffu, any)) continue;
       PH_BEGIN(t_expn);
       // EXPN: items waiting on a newly completed nonterminal
-      for (int w = wl_lane(); w < W; w += 32) {
-        uint32_t acc = 0;
-        for (int v = 0; v < VW; ++v) {
-          uint32_t nw = sh.nt[v];
-          while (nw) {
-            int b = __ffs(nw) - 1;
-            nw &= nw - 1;
-            acc |= g.exp_nt[(size_t)((v << 5) + b) * W + w];
-          }
-        }
-        sh.expn[w] = acc;
-      }
+      expn_of_set(g, sh.nt, sh.expn);
       __syncwarp();
       PH_END(5, t_expn);
       PH_BEGIN(t_part);
