@@ -194,7 +194,6 @@ def main():
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # > 129 MB L2
     stream = torch.cuda.current_stream()
     checks = w.B * w.k * w.K
-    launches_per_step = 5  # validate, pick, select_spec, select, commit
 
     def step(xbuf):
         epic.validate_batch(g, t, xbuf, pos, cand, valid)
@@ -230,6 +229,11 @@ def main():
     step_ms = [a.elapsed_time(c) for a, b, c in ev]
     val_ms = [a.elapsed_time(b) for a, b, c in ev]
     st = t.stats()
+    region = st['region_checks'] > 0
+    # kernels of the timed region: validate's own (one walk kernel, or the
+    # forward chart, good masks and region checks) + pick + two selection
+    # kernels + commit
+    launches = st['validate_kernels'] + 4 * args.steps
     ms = float(np.mean(step_ms))
     vms = float(np.mean(val_ms))
     if world > 1:
@@ -275,7 +279,9 @@ def main():
     roof = {'bound': 'alu', 'achieved': achieved, 'peak': int_peak, 'unit': 'T word-ops/s',
             'frac': achieved / int_peak, 'traffic': None,
             'peak_source': 'derived: %s (%s sm_max_mhz)' % (INT_PEAK_NOTE, pk_kind),
-            'kernel': 'k_validate_warp', 'kernel_ms': vms}
+            'kernel': ('k_forward + k_good + k_check (epic_validate_batch, by region)' if region
+                       else 'k_validate_warp'),
+            'kernel_ms': vms}
     line = {'metric': 'candidate validity checks/sec', 'value': value, 'unit': 'checks/s',
             'n_gpus': world, 'steps': args.steps, 'warmup': args.warmup, 'ms_per_step': ms,
             'higher_is_better': True, 'scaling': 'weak', 'vs_baseline': None, 'dtype': 'int32',
@@ -285,7 +291,7 @@ def main():
                        'parallelism': 'replicas' if world > 1 else 'single'},
             'step_latency_us': ms * 1e3, 'validate_checks_per_s': total_checks / (vms / 1e3),
             'valid_fraction': st['valid'] / max(1, st['checks']), 'overflow': st['overflow'],
-            'gpu_launches': launches_per_step * args.steps,
+            'gpu_launches': int(launches), 'validate_path': 'region' if region else 'walk',
             'e2e': {'value': total_checks / (e2e_step / 1e3), 'unit': 'checks/s', 'h2d_bytes_per_step': int(h2d),
                     'd2h_bytes_per_step': int(d2h)},
             'roofline': roof, 'clocks': clk.summary()}

@@ -218,6 +218,9 @@ typedef struct {
   uint64_t cover_checks;     /* regular-cover group tests (Alg. 4 line 9)      */
   uint64_t exact_checks;     /* joint exact checks (Alg. 4 line 21)            */
   uint64_t selected;         /* candidates committed by selection              */
+  uint64_t region_checks;    /* of the checks, those answered by region walks
+                                over a per-sequence forward chart            */
+  uint64_t validate_kernels; /* kernel launches made by epic_validate_batch*  */
 } epic_stats;
 
 /* Copy the counters (synchronizes the lexer table's last stream); out_bytes

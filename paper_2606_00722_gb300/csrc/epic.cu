@@ -576,6 +576,7 @@ struct epic_lexer_table {
   WsDims dims{};
   int ctas = 0;
   unsigned long long* d_stats = nullptr;
+  mutable unsigned long long n_region = 0, n_vkernels = 0;  // host-side counters
   unsigned long long* d_counter = nullptr;
   int8_t* d_spec = nullptr;  // speculative Alg. 4 answers, 2 per sequence
   char* d_seq = nullptr;     // per-sequence forward charts (region checks)
@@ -794,14 +795,17 @@ epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const in
     if (sm && wpc >= 1) {
       size_t dyn = per * wpc;
       cudaFuncSetAttribute(k_forward<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-      k_forward<true><<<(B + wpc - 1) / wpc, 32 * wpc, dyn, st>>>(dg, t->d_table, t->vocab, d_x, B, n, sp, rmax);
+      k_forward<true><<<(B + wpc - 1) / wpc, 32 * wpc, dyn, st>>>(dg, t->d_table, t->vocab, d_x, B, n, sp, rmax,
+                                                                    t->d_stats);
     } else {
       k_forward<false><<<(B + kWarpsPerCta - 1) / kWarpsPerCta, 32 * kWarpsPerCta, 0, st>>>(
-          dg, t->d_table, t->vocab, d_x, B, n, sp, 0);
+          dg, t->d_table, t->vocab, d_x, B, n, sp, 0, t->d_stats);
     }
   }
   // 2. good masks
   k_good<<<B, 32 * kGoodWarps, 0, st>>>(dg, B, sp);
+  t->n_region += total;
+  t->n_vkernels += 3;
   // 3. checks
   cudaMemsetAsync(t->d_counter, 0, 8, st);
   size_t per = smem_per_warp(wp.nmax, rmax, dg.W, dg.VW);
@@ -1101,6 +1105,7 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
   // spread the walks over every SM: no more warps per CTA than walks per SM
   int per_sm = (int)((t->wwarps + sm_count() - 1) / sm_count());
   if (wpc > per_sm) wpc = std::max(2, per_sm);
+  t->n_vkernels += 1;
   if (wpc >= 2) {
     size_t dyn = per * wpc + (gsm ? gt : 0);
     int blocks = (t->wwarps + wpc - 1) / wpc;
@@ -1170,6 +1175,7 @@ epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_
   int wpc = (W > 32) ? 0 : (int)std::min<size_t>(kWarpsPerCta, smem_cap / sper);
   unsigned long long* counter = (unsigned long long*)base;
   if (cudaMemsetAsync(counter, 0, sizeof(unsigned long long), st) != cudaSuccess) return EPIC_ERR_CUDA;
+  t->n_vkernels += 1;
   if (wpc >= 2) {
     long long warps = std::min<long long>({total, fit, (long long)sm_count() * 2 * kWarpsPerCta});
     int per_cta = (int)std::min<long long>(wpc, warps);
@@ -1257,7 +1263,13 @@ epic_status epic_get_stats(const epic_lexer_table* t, epic_stats* out, size_t ou
   out->cover_checks = h[S_COVER];
   out->exact_checks = h[S_EXACT];
   out->selected = h[S_SELECTED];
-  if (reset && cudaMemset(t->d_stats, 0, sizeof(h)) != cudaSuccess) return EPIC_ERR_CUDA;
+  out->region_checks = t->n_region;
+  out->validate_kernels = t->n_vkernels;
+  if (reset) {
+    if (cudaMemset(t->d_stats, 0, sizeof(h)) != cudaSuccess) return EPIC_ERR_CUDA;
+    t->n_region = 0;
+    t->n_vkernels = 0;
+  }
   return EPIC_OK;
 }
 

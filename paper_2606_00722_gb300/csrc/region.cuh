@@ -114,7 +114,8 @@ enum { M_NCOLS = 0, M_NEDGES = 1, M_START = 2, M_ACCEPT = 3, M_STATUS = 4, M_NEN
 template <bool SM>
 __global__ void __launch_bounds__(32 * kWarpsPerCta) k_forward(DevGrammar g, const LexEntry* __restrict__ table,
                                                                 int vocab, const int32_t* __restrict__ x, int B, int n,
-                                                                SeqPack sp, int rmax) {
+                                                                SeqPack sp, int rmax,
+                                                                unsigned long long* stats) {
   __shared__ WSh shm[kWarpsPerCta];
   extern __shared__ __align__(16) unsigned char dyn[];
   int warp = threadIdx.x >> 5;
@@ -161,6 +162,8 @@ __global__ void __launch_bounds__(32 * kWarpsPerCta) k_forward(DevGrammar g, con
     rec.meta[M_START] = walk.start_col;
     rec.meta[M_STATUS] = r == 1 ? 1 : (r == 0 ? 0 : -1);
     rec.meta[M_NENT] = (int)walk.nent;
+    atomicAdd(&stats[4], (unsigned long long)walk.ncols);  // columns and entries of the forward charts
+    atomicAdd(&stats[5], (unsigned long long)walk.nent);
   }
 }
 
@@ -198,8 +201,9 @@ __global__ void __launch_bounds__(32 * kGoodWarps) k_good(DevGrammar g, int B, S
   const int32_t* col = a.ws.col_off;
   const int32_t* org = a.ws.org;
   const int start = meta[M_START], accept = meta[M_ACCEPT];
-  __shared__ int s_flag;
+  __shared__ int s_flag, s_self;
   __shared__ uint32_t s_nt[kGoodWarps][kWMaxVW];
+  constexpr int KW = kWMaxW / 32;  // item words per lane
   int32_t* cur_o = a.cursor;          // [N + 1]
   int32_t* cur_s = a.cursor + N + 1;  // [N + 1]
   // edges by source and entries by origin (CSR), entry index by (column, origin)
@@ -249,9 +253,12 @@ __global__ void __launch_bounds__(32 * kGoodWarps) k_good(DevGrammar g, int B, S
     const long long k0 = col[j], k1 = col[j + 1];
     if (k0 == k1) continue;
     // EXPN of what completes from origin j at each column j2 (j2 = j included)
-    int self_si = -1;
-    for (int si = s0; si < s1; ++si)
-      if (a.succ_idx[si] == j) self_si = si - s0;
+    if (tid == 0) s_self = -1;
+    __syncthreads();
+    for (int si = s0 + tid; si < s1; si += nthr)
+      if (a.succ_idx[si] == j) s_self = si - s0;
+    __syncthreads();
+    const int self_si = s_self;
     for (int si = s0 + warp; si < s1; si += kGoodWarps) {
       const int j2 = a.succ_idx[si];
       const uint32_t* cn = a.rec.cnt + (size_t)a.eidx[tri_index(j2, j)] * VW;
@@ -259,43 +266,80 @@ __global__ void __launch_bounds__(32 * kGoodWarps) k_good(DevGrammar g, int B, S
     }
     __syncthreads();
     // from the later columns: scans along the out-edges, nested constituents
+    // (the lanes look up 32 successor columns at a time)
     for (long long k = k0 + warp; k < k1; k += kGoodWarps) {
       const int o = org[k];
       const uint32_t* bits = a.ws.bits + (size_t)k * W;
       uint32_t* Gk = G + (size_t)k * W;
-      bool nz = false;
-      for (int w = lane; w < W; w += 32) {
-        uint32_t acc = 0;
-        if (j == accept && o == start && w == (g.accept_item >> 5)) acc |= 1u << (g.accept_item & 31);
-        for (int ei = a.out_off[j]; ei < a.out_off[j + 1]; ++ei) {
-          const int e = a.out_idx[ei];
-          const int k2 = a.eidx[tri_index(a.rec.e_dst[e], o)];
-          if (k2 < 0 || !a.gnz[k2]) continue;
-          const uint32_t* G2 = G + (size_t)k2 * W;
-          const uint32_t* L = a.rec.e_lbl + (size_t)e * 8;
-          uint32_t m = 0;
-          bool eps = true;
-          for (int lw = 0; lw < 8; ++lw) {
-            uint32_t lm = L[lw];
-            eps &= lm == 0;
-            while (lm) {
-              const int bb = __ffs(lm) - 1;
-              lm &= lm - 1;
-              const int t = (lw << 5) + bb;
-              if (t < g.T) m |= g.exp_term[(size_t)t * W + w];
+      uint32_t acc[KW];
+#pragma unroll
+      for (int i = 0; i < KW; ++i) acc[i] = 0;
+      if (j == accept && o == start && lane == ((g.accept_item >> 5) & 31))
+        acc[g.accept_item >> 10] |= 1u << (g.accept_item & 31);
+      for (int ei = a.out_off[j]; ei < a.out_off[j + 1]; ++ei) {
+        const int e = a.out_idx[ei];
+        const int k2 = a.eidx[tri_index(a.rec.e_dst[e], o)];
+        if (k2 < 0 || !a.gnz[k2]) continue;
+        const uint32_t* G2 = G + (size_t)k2 * W;
+        const uint32_t* L = a.rec.e_lbl + (size_t)e * 8;
+        uint32_t lw8[8];
+        bool eps = true;
+        for (int lw = 0; lw < 8; ++lw) {
+          lw8[lw] = L[lw];
+          eps &= lw8[lw] == 0;
+        }
+#pragma unroll
+        for (int i = 0; i < KW; ++i) {
+          const int w = lane + 32 * i;
+          if (w < W) {
+            if (eps) {
+              acc[i] |= G2[w];
+            } else {
+              uint32_t m = 0;
+              for (int lw = 0; lw < 8; ++lw) {
+                uint32_t lm = lw8[lw];
+                while (lm) {
+                  const int bb = __ffs(lm) - 1;
+                  lm &= lm - 1;
+                  const int t = (lw << 5) + bb;
+                  if (t < g.T) m |= g.exp_term[(size_t)t * W + w];
+                }
+              }
+              acc[i] |= m & shr1_word(G2, w, W);
             }
           }
-          acc |= eps ? G2[w] : (m & shr1_word(G2, w, W));
         }
-        for (int si = s0; si < s1; ++si) {
-          if (si - s0 == self_si) continue;
-          const int k3 = a.eidx[tri_index(a.succ_idx[si], o)];
-          if (k3 < 0 || !a.gnz[k3]) continue;
-          acc |= a.expn[(size_t)(si - s0) * W + w] & shr1_word(G + (size_t)k3 * W, w, W);
+      }
+      for (int sb = s0; sb < s1; sb += 32) {
+        const int si = sb + lane;
+        int k3 = -1;
+        if (si < s1 && si - s0 != self_si) {
+          const int kk = a.eidx[tri_index(a.succ_idx[si], o)];
+          if (kk >= 0 && a.gnz[kk]) k3 = kk;
         }
-        const uint32_t v = bits[w] & acc;
-        Gk[w] = v;
-        nz |= v != 0;
+        unsigned act = __ballot_sync(0xffffffffu, k3 >= 0);
+        while (act) {
+          const int l = __ffs(act) - 1;
+          act &= act - 1;
+          const int kk = __shfl_sync(0xffffffffu, k3, l);
+          const uint32_t* ex = a.expn + (size_t)(sb + l - s0) * W;
+          const uint32_t* G3 = G + (size_t)kk * W;
+#pragma unroll
+          for (int i = 0; i < KW; ++i) {
+            const int w = lane + 32 * i;
+            if (w < W) acc[i] |= ex[w] & shr1_word(G3, w, W);
+          }
+        }
+      }
+      bool nz = false;
+#pragma unroll
+      for (int i = 0; i < KW; ++i) {
+        const int w = lane + 32 * i;
+        if (w < W) {
+          const uint32_t v = bits[w] & acc[i];
+          Gk[w] = v;
+          nz |= v != 0;
+        }
       }
       nz = __any_sync(0xffffffffu, nz);
       if (lane == 0) a.gnz[k] = nz ? 1 : 0;
@@ -319,19 +363,29 @@ __global__ void __launch_bounds__(32 * kGoodWarps) k_good(DevGrammar g, int B, S
         for (int round = 0; round <= W * 32; ++round) {
           for (int v = lane; v < VW; v += 32) bset[v] = 0;
           __syncwarp();
-          for (long long kp = col[o]; kp < col[o + 1]; ++kp) {
-            const int o2 = org[kp];
-            const long long kk = (o2 == o) ? k : a.eidx[tri_index(j, o2)];
-            if (kk < 0 || (kk != k && !a.gnz[kk])) continue;
-            const uint32_t* P = a.ws.bits + (size_t)kp * W;
-            const uint32_t* GK = G + (size_t)kk * W;
-            for (int w = lane; w < W; w += 32) {
-              uint32_t m = P[w] & g.any_nt[w] & shr1_word(GK, w, W);
-              while (m) {
-                const int bb = __ffs(m) - 1;
-                m &= m - 1;
-                const int Bn = g.item_next[(w << 5) + bb] - g.T;
-                atomicOr(&bset[Bn >> 5], 1u << (Bn & 31));
+          for (long long kb = col[o]; kb < col[o + 1]; kb += 32) {  // 32 lookups at a time
+            const long long kp = kb + lane;
+            long long kk = -1;
+            if (kp < col[o + 1]) {
+              const int o2 = org[kp];
+              kk = (o2 == o) ? k : a.eidx[tri_index(j, o2)];
+              if (kk >= 0 && kk != k && !a.gnz[kk]) kk = -1;
+            }
+            unsigned act = __ballot_sync(0xffffffffu, kk >= 0);
+            while (act) {
+              const int l = __ffs(act) - 1;
+              act &= act - 1;
+              const long long kq = __shfl_sync(0xffffffffu, kk, l);
+              const uint32_t* P = a.ws.bits + (size_t)(kb + l) * W;
+              const uint32_t* GK = G + (size_t)kq * W;
+              for (int w = lane; w < W; w += 32) {
+                uint32_t m = P[w] & g.any_nt[w] & shr1_word(GK, w, W);
+                while (m) {
+                  const int bb = __ffs(m) - 1;
+                  m &= m - 1;
+                  const int Bn = g.item_next[(w << 5) + bb] - g.T;
+                  atomicOr(&bset[Bn >> 5], 1u << (Bn & 31));
+                }
               }
             }
           }
@@ -612,6 +666,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerCta) k_check(
     const int32_t* xb = x + b * n;
     int i = pos[b * k + jj], t = cand[jb];
     int r;
+    long long own_cols = 0, own_ent = 0;  // columns and entries this check stored
     if (i < 0 || i >= n || xb[i] >= 0 || t < 0 || t >= vocab) {
       r = -2;
     } else {
@@ -623,11 +678,15 @@ __global__ void __launch_bounds__(32 * kWarpsPerCta) k_check(
         RegionCheck<SM> rc{walk, a, rs.fmap, rs.act, rs.act_f};
         r = rc.run(xb, n, i, t);
         if (r < 0) walk.cleanup();
+        own_cols = walk.ncols - walk.base_cols;
+        own_ent = walk.nent;
       } else {  // the sequence's forward chart did not fit: walk the whole check
         walk.base_cols = 0;
         walk.base_ent = 0;
         walk.suffix_mode = false;
         r = walk.run(xb, n, i, t);
+        own_cols = walk.ncols;
+        own_ent = walk.nent;
       }
       walk.base_cols = 0;
       walk.base_ent = 0;
@@ -638,8 +697,8 @@ __global__ void __launch_bounds__(32 * kWarpsPerCta) k_check(
     n_valid += r == 1;
     n_ovf += r == -1;
     n_bad += r == -2;
-    n_cols += walk.ncols;
-    n_ent += walk.nent;
+    n_cols += own_cols;
+    n_ent += own_ent;
   }
   if (lane == 0 && n_checks) {
     atomicAdd(&stats[0], n_checks);

@@ -48,7 +48,8 @@ def build(force: bool = False, verbose: bool = False) -> str:
 
 class _Stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in ('checks', 'valid', 'overflow', 'bad_inputs', 'columns',
-                                          'entries', 'cover_checks', 'exact_checks', 'selected')]
+                                          'entries', 'cover_checks', 'exact_checks', 'selected',
+                                          'region_checks', 'validate_kernels')]
 
 
 class _Desc(C.Structure):
