@@ -136,7 +136,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerCta) k_forward(DevGrammar g, con
   for (size_t w = threadIdx.x & 31; w < (size_t)sp.nmax * g.W; w += 32) a.ws.stage[w] = 0;
   for (size_t w = threadIdx.x & 31; w < (size_t)sp.nmax * g.VW; w += 32) a.ws.bdone[w] = 0;
   __syncwarp();
-  WarpWalker<SM> walk(g, table, a.ws, sh, sp.nmax, sp.emax, vocab);
+  WarpWalker<SM, true> walk(g, table, a.ws, sh, sp.nmax, sp.emax, vocab);
   if constexpr (SM) {
     size_t per = smem_per_warp(sp.nmax, rmax, g.W, g.VW);
     unsigned char* base = dyn + per * warp;
@@ -427,7 +427,7 @@ __global__ void __launch_bounds__(32 * kGoodWarps) k_good(DevGrammar g, int B, S
 // ------------------------------------------------------------------ 3. checks by region
 template <bool SM>
 struct RegionCheck {
-  WarpWalker<SM>& w;
+  WarpWalker<SM, true>& w;
   SeqArena& a;
   int32_t* fmap;     // [nmax] F node -> own column with carried rows (-1)
   int32_t* act;      // [nmax] own columns whose rows wait on nonterminals
@@ -640,7 +640,7 @@ __global__ void __launch_bounds__(32 * kWarpsPerCta) k_check(
   }
   __syncwarp();
   const long long gw = (long long)blockIdx.x * (blockDim.x >> 5) + warp;
-  WarpWalker<SM> walk(g, table, wp.carve(gw), sh, wp.nmax, wp.emax, vocab);
+  WarpWalker<SM, true> walk(g, table, wp.carve(gw), sh, wp.nmax, wp.emax, vocab);
   if constexpr (SM) {
     size_t per = smem_per_warp(wp.nmax, rmax, g.W, g.VW);
     unsigned char* base = dyn + per * warp;

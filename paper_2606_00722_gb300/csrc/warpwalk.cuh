@@ -121,8 +121,10 @@ __device__ unsigned long long g_phase[16];
 
 // SM = true keeps the rows of the column under construction in shared memory
 // (slot-mapped, rmax rows); SM = false keeps them in the per-warp global
-// stage.  KWv item words per lane: rows of up to 32 KWv words.
-template <bool SM, int KWv = (SM ? 1 : kWMaxW / 32)>
+// stage.  KWv item words per lane: rows of up to 32 KWv words.  EXT = true
+// adds the base chart, the suffix mode and the recording of checks by region
+// (compiled out of whole-graph walks).
+template <bool SM, bool EXT = false, int KWv = (SM ? 1 : kWMaxW / 32)>
 class WarpWalker {
   static constexpr int KW = KWv;  // item words per lane
 
@@ -224,16 +226,23 @@ class WarpWalker {
 
   // ------------------------------------------------------------ chart access
   __device__ long long cbeg(int c) const {
+    if constexpr (!EXT) return ws.col_off[c];
     return c < base_cols ? (long long)b_col_off[c] : base_ent + ws.col_off[c - base_cols];
   }
   __device__ long long cend(int c) const {
+    if constexpr (!EXT) return ws.col_off[c + 1];
     return c < base_cols ? (long long)b_col_off[c + 1] : base_ent + ws.col_off[c - base_cols + 1];
   }
-  __device__ int eorg(long long k) const { return k < base_ent ? b_org[k] : ws.org[k - base_ent]; }
+  __device__ int eorg(long long k) const {
+    if constexpr (!EXT) return ws.org[k];
+    return k < base_ent ? b_org[k] : ws.org[k - base_ent];
+  }
   __device__ const uint32_t* ebits(long long k) const {
+    if constexpr (!EXT) return ws.bits + (size_t)k * W;
     return k < base_ent ? b_bits + (size_t)k * W : ws.bits + (size_t)(k - base_ent) * W;
   }
   __device__ uint32_t esum(long long k, int which) const {
+    if constexpr (!EXT) return ws.esum[(size_t)k * 2 + which];
     return k < base_ent ? b_esum[(size_t)k * 2 + which] : ws.esum[(size_t)(k - base_ent) * 2 + which];
   }
 
@@ -412,7 +421,7 @@ class WarpWalker {
   __device__ void scatter(int col, const uint32_t* M, bool shift, int which, uint32_t fold) {
     const int lane = wl_lane();
     const long long b = cbeg(col), e = cend(col);
-    if (W > 16) {  // wide rows: the lanes share each entry's words
+    if (!SM && W > 16) {  // wide rows in the global stage: the lanes share each entry's words
       for (long long base = b; base < e; base += 32) {
         const long long k = base + lane;
         const bool act = k < e && (which < 0 || (esum(k, which) & fold) != 0);
@@ -561,7 +570,8 @@ class WarpWalker {
     rec->n_edges = __shfl_sync(0xffffffffu, rec->n_edges, 0);
   }
   __device__ void arrive_inner(int src, const uint32_t* M, bool shift) {
-    if (rec) record_edge(src, shift);
+    if constexpr (EXT)
+      if (rec) record_edge(src, shift);
     if (shift)
       scatter(src, M, true, 1, label_fold);
     else
@@ -601,7 +611,7 @@ class WarpWalker {
         return;
       }
       int o = bm_highest(sh.dirty, c + 1);
-      if (suffix_mode) {
+      if (EXT && suffix_mode) {
         if (o < 0) break;
         if (o < base_cols) {  // resolved by the good masks at finish
           if (wl_lane() == 0) sh.dirty[o >> 5] &= ~(1u << (o & 31));
@@ -686,7 +696,7 @@ class WarpWalker {
       bool nz = false;
       for (int w = wl_lane(); w < W; w += 32) nz |= row[w] != 0;
       nz = __any_sync(0xffffffffu, nz);
-      if (nz && suffix_mode && o < base_cols) {
+      if (EXT && nz && suffix_mode && o < base_cols) {
         long long kf = find_base(res_node, o);
         bool hit = false;
         if (kf >= 0)
@@ -694,7 +704,7 @@ class WarpWalker {
         if (__any_sync(0xffffffffu, hit)) found = 1;
         nz = false;  // not kept
       }
-      if (nz && suffix_mode && o == region_start && res_node == accept_node &&
+      if (EXT && nz && suffix_mode && o == region_start && res_node == accept_node &&
           ((row[g.accept_item >> 5] >> (g.accept_item & 31)) & 1u))
         found = 1;
       if (nz) {
@@ -709,7 +719,7 @@ class WarpWalker {
           }
           uint32_t* dst = ws.bits + (size_t)E * W;
           for (int w = wl_lane(); w < W; w += 32) dst[w] = row[w];
-          if (rec) {  // completed nonterminals of the entry
+          if (EXT && rec) {  // completed nonterminals of the entry
             for (int v = wl_lane(); v < VW; v += 32) sh.nt[v] = 0;
             __syncwarp();
             row_nts(row, g.complete, true, sh.nt);
@@ -731,7 +741,7 @@ class WarpWalker {
     }
     if (wl_lane() == 0) {
       ws.col_off[oc + 1] = (int)E;
-      if (rec) rec->col_gap[c] = cur_gap ? 1 : 0;
+      if (EXT && rec) rec->col_gap[c] = cur_gap ? 1 : 0;
     }
     __syncwarp();
     nent = E;
@@ -1034,7 +1044,7 @@ class WarpWalker {
         close_column(c, true);
         finish_column(c);
         if (status) return -1;
-        if (rec) {
+        if (EXT && rec) {
           rec_range(rec->gap_col, i, j, c);
           if (span_lo >= 0) rec_range(rec->post_col, span_lo, span_hi, c);
         }
@@ -1056,7 +1066,7 @@ class WarpWalker {
           src = prev_gap;
         }
         frontier_from(src, first);
-        if (rec) rec_range(rec->pre_col, i, j, src);
+        if (EXT && rec) rec_range(rec->pre_col, i, j, src);
         span_lo = i;
         span_hi = j;
         for (int p = i; p < j && nf > 0; ++p) {
@@ -1071,7 +1081,7 @@ class WarpWalker {
           close_column(c, false);
           finish_column(c);
           if (status) return -1;
-          if (rec) {
+          if (EXT && rec) {
             rec_range(rec->post_col, i, j, c);
             if (wl_lane() == 0) rec->meta[3] = c;
           }
@@ -1081,7 +1091,7 @@ class WarpWalker {
       first = false;
       i = j;
     }
-    if (rec && wl_lane() == 0) rec->meta[3] = prev_gap;
+    if (EXT && rec && wl_lane() == 0) rec->meta[3] = prev_gap;
     return accepts(prev_gap, start_col) ? 1 : 0;
   }
 };

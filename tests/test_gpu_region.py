@@ -105,3 +105,15 @@ def test_wide_grammars_by_region(cuda, name, seed, kw):
     assert st['overflow'] == 0
     ref = oracle.Oracle(w.grammar, w.vocab).validate_batch(w.x, w.pos, w.cand, nthreads=NTHREADS)
     np.testing.assert_array_equal(got, ref)
+
+
+def test_clike_full_length_row(cuda):
+    """clike-512 at its full row length (512 tokens) on one row, 4 positions x
+    8 candidates, by region (the default for its item width), against the
+    oracle."""
+    w = make_workload('clike-512', 44, batch=1, k=4, K=8)
+    got, st = run_gpu(w.grammar, w.vocab, w.x, w.pos, w.cand, cuda)
+    assert st['overflow'] == 0
+    assert st['region_checks'] == w.cand.size
+    ref = oracle.Oracle(w.grammar, w.vocab).validate_batch(w.x, w.pos, w.cand, nthreads=NTHREADS)
+    np.testing.assert_array_equal(got, ref)
