@@ -189,7 +189,7 @@ constexpr int kGoodWarps = 32;  // one CTA per sequence
 //    waiting on B has its advanced item good at (j, o2).
 // The first three read later columns only (final); the last two read this
 // column: its entries iterate to the least fixpoint together.
-__global__ void __launch_bounds__(32 * kGoodWarps) k_good(DevGrammar g, int B, SeqPack sp) {
+__global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B, SeqPack sp) {
   const long long b = blockIdx.x;
   if (b >= B) return;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nthr = blockDim.x;
@@ -247,6 +247,8 @@ __global__ void __launch_bounds__(32 * kGoodWarps) k_good(DevGrammar g, int B, S
   __syncthreads();
 
   uint32_t* G = a.good;
+  uint32_t* sfold = (uint32_t*)a.cursor;  // per successor of the column (the cursors are free now)
+  const int nwl = (W + 31) >> 5;          // item words per lane in use
   for (int j = N - 1; j >= 0; --j) {
     const int s0 = a.succ_off[j], s1 = a.succ_off[j + 1];
     const bool gap = a.rec.col_gap[j] != 0;
@@ -263,6 +265,11 @@ __global__ void __launch_bounds__(32 * kGoodWarps) k_good(DevGrammar g, int B, S
       const int j2 = a.succ_idx[si];
       const uint32_t* cn = a.rec.cnt + (size_t)a.eidx[tri_index(j2, j)] * VW;
       expn_of_set(g, cn, a.expn + (size_t)(si - s0) * W);
+      if (lane == 0) {  // folded set (bit C mod 32): a filter against an entry's waited nonterminals
+        uint32_t f = 0;
+        for (int v = 0; v < VW; ++v) f |= cn[v];
+        sfold[si - s0] = f;
+      }
     }
     __syncthreads();
     // from the later columns: scans along the out-edges, nested constituents
@@ -290,6 +297,7 @@ __global__ void __launch_bounds__(32 * kGoodWarps) k_good(DevGrammar g, int B, S
         }
 #pragma unroll
         for (int i = 0; i < KW; ++i) {
+          if (i >= nwl) break;
           const int w = lane + 32 * i;
           if (w < W) {
             if (eps) {
@@ -310,10 +318,11 @@ __global__ void __launch_bounds__(32 * kGoodWarps) k_good(DevGrammar g, int B, S
           }
         }
       }
+      const uint32_t wfold = a.ws.esum[(size_t)k * 2];  // waited nonterminals, folded
       for (int sb = s0; sb < s1; sb += 32) {
         const int si = sb + lane;
         int k3 = -1;
-        if (si < s1 && si - s0 != self_si) {
+        if (si < s1 && si - s0 != self_si && (sfold[si - s0] & wfold) != 0) {
           const int kk = a.eidx[tri_index(a.succ_idx[si], o)];
           if (kk >= 0 && a.gnz[kk]) k3 = kk;
         }
@@ -326,6 +335,7 @@ __global__ void __launch_bounds__(32 * kGoodWarps) k_good(DevGrammar g, int B, S
           const uint32_t* G3 = G + (size_t)kk * W;
 #pragma unroll
           for (int i = 0; i < KW; ++i) {
+            if (i >= nwl) break;
             const int w = lane + 32 * i;
             if (w < W) acc[i] |= ex[w] & shr1_word(G3, w, W);
           }
