@@ -65,3 +65,16 @@ def test_host_side_argument_errors():
     # empty batches are no-ops that touch nothing
     assert lib.epic_commit(None, 0, 5, None, 3, None, None, None) == 0
     assert lib.epic_pick_candidates(None, None, None, 0, 4, 4, None, None, None) == 0
+
+
+def test_stats_struct_matches_header():
+    """The binding's epic_stats mirror has the header's fields, in order, all
+    uint64 (the library copies the whole struct)."""
+    src = open(os.path.join(ROOT, 'include', 'epic.h')).read()
+    body = re.search(r'typedef struct \{(.*?)\} epic_stats;', src, flags=re.S).group(1)
+    body = re.sub(r'/\*.*?\*/', '', body, flags=re.S)
+    fields = re.findall(r'uint64_t\s+(\w+)\s*;', body)
+    from paper_2606_00722_gb300.epic import _Stats
+    assert [f for f, _ in _Stats._fields_] == fields
+    import ctypes
+    assert ctypes.sizeof(_Stats) == 8 * len(fields)
