@@ -176,7 +176,6 @@ __device__ __forceinline__ uint32_t shr1_word(const uint32_t* src, int w, int W)
 }
 
 constexpr int kGoodWarps = 32;  // one CTA per sequence
-constexpr int kGoodSerial = 96;  // columns with at most this many entries settle on one warp
 
 // Good items of a sequence's forward chart, columns from last to first.
 // Item i of entry (j, o) is good when it is present and
@@ -356,81 +355,7 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
       if (lane == 0) a.gnz[k] = nz ? 1 : 0;
     }
     __syncthreads();
-    // completions within the column and the self rules, to the fixpoint.
-    // An entry's completions read only entries of this column with a lower
-    // origin (the origins of column o are <= o), so one ascending pass settles
-    // the column if each entry is iterated to its own fixpoint.
-    uint32_t* bset = s_nt[warp];
-    auto settle = [&](long long k) -> bool {  // warp: iterate entry k; true if it changed
-      const int o = org[k];
-      const uint32_t* bits = a.ws.bits + (size_t)k * W;
-      uint32_t* Gk = G + (size_t)k * W;
-      bool changed = false;
-      // each round that changes the entry adds an item
-      for (int round = 0; round <= W * 32; ++round) {
-        for (int v = lane; v < VW; v += 32) bset[v] = 0;
-        __syncwarp();
-        for (long long kb = col[o]; kb < col[o + 1]; kb += 32) {  // 32 lookups at a time
-          const long long kp = kb + lane;
-          long long kk = -1;
-          if (kp < col[o + 1]) {
-            const int o2 = org[kp];
-            kk = (o2 == o) ? k : a.eidx[tri_index(j, o2)];
-            if (kk >= 0 && kk != k && !a.gnz[kk]) kk = -1;
-          }
-          unsigned act = __ballot_sync(0xffffffffu, kk >= 0);
-          while (act) {
-            const int l = __ffs(act) - 1;
-            act &= act - 1;
-            const long long kq = __shfl_sync(0xffffffffu, kk, l);
-            const uint32_t* P = a.ws.bits + (size_t)(kb + l) * W;
-            const uint32_t* GK = G + (size_t)kq * W;
-            for (int w = lane; w < W; w += 32) {
-              uint32_t m = P[w] & g.any_nt[w] & shr1_word(GK, w, W);
-              while (m) {
-                const int bb = __ffs(m) - 1;
-                m &= m - 1;
-                const int Bn = g.item_next[(w << 5) + bb] - g.T;
-                atomicOr(&bset[Bn >> 5], 1u << (Bn & 31));
-              }
-            }
-          }
-        }
-        __syncwarp();
-        bool ch = false;
-        for (int w = lane; w < W; w += 32) {
-          uint32_t add = 0;
-          uint32_t m = bits[w] & g.complete[w];
-          while (m) {
-            const int bb = __ffs(m) - 1;
-            m &= m - 1;
-            const int L2 = g.item_lhs[(w << 5) + bb];
-            if ((bset[L2 >> 5] >> (L2 & 31)) & 1u) add |= 1u << bb;
-          }
-          const uint32_t s = shr1_word(Gk, w, W);
-          if (gap) add |= g.next_any[w] & s;
-          if (self_si >= 0) add |= a.expn[(size_t)self_si * W + w] & s;
-          add &= bits[w];
-          const uint32_t old = Gk[w];
-          if ((old | add) != old) {
-            Gk[w] = old | add;
-            ch = true;
-          }
-        }
-        if (!__any_sync(0xffffffffu, ch)) break;
-        changed = true;
-        if (lane == 0) a.gnz[k] = 1;
-        __syncwarp();
-      }
-      return changed;
-    };
-    if (k1 - k0 <= kGoodSerial) {  // small column: one warp, ascending origins
-      if (warp == 0)
-        for (long long k = k0; k < k1; ++k) settle(k);
-      __syncthreads();
-      continue;
-    }
-    // large column: all warps, passes until none changes anything
+    // completions within the column and the self rules, to the fixpoint
     for (int pass = 0;; ++pass) {
       if (pass > (1 << 20)) {  // cannot happen before the fixpoint; never silently wrong
         if (tid == 0) meta[M_STATUS] = -1;
@@ -439,7 +364,67 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
       if (tid == 0) s_flag = 0;
       __syncthreads();
       bool changed = false;
-      for (long long k = k0 + warp; k < k1; k += kGoodWarps) changed |= settle(k);
+      uint32_t* bset = s_nt[warp];
+      for (long long k = k0 + warp; k < k1; k += kGoodWarps) {
+        const int o = org[k];
+        const uint32_t* bits = a.ws.bits + (size_t)k * W;
+        uint32_t* Gk = G + (size_t)k * W;
+        // each round that changes the entry adds an item
+        for (int round = 0; round <= W * 32; ++round) {
+          for (int v = lane; v < VW; v += 32) bset[v] = 0;
+          __syncwarp();
+          for (long long kb = col[o]; kb < col[o + 1]; kb += 32) {  // 32 lookups at a time
+            const long long kp = kb + lane;
+            long long kk = -1;
+            if (kp < col[o + 1]) {
+              const int o2 = org[kp];
+              kk = (o2 == o) ? k : a.eidx[tri_index(j, o2)];
+              if (kk >= 0 && kk != k && !a.gnz[kk]) kk = -1;
+            }
+            unsigned act = __ballot_sync(0xffffffffu, kk >= 0);
+            while (act) {
+              const int l = __ffs(act) - 1;
+              act &= act - 1;
+              const long long kq = __shfl_sync(0xffffffffu, kk, l);
+              const uint32_t* P = a.ws.bits + (size_t)(kb + l) * W;
+              const uint32_t* GK = G + (size_t)kq * W;
+              for (int w = lane; w < W; w += 32) {
+                uint32_t m = P[w] & g.any_nt[w] & shr1_word(GK, w, W);
+                while (m) {
+                  const int bb = __ffs(m) - 1;
+                  m &= m - 1;
+                  const int Bn = g.item_next[(w << 5) + bb] - g.T;
+                  atomicOr(&bset[Bn >> 5], 1u << (Bn & 31));
+                }
+              }
+            }
+          }
+          __syncwarp();
+          bool ch = false;
+          for (int w = lane; w < W; w += 32) {
+            uint32_t add = 0;
+            uint32_t m = bits[w] & g.complete[w];
+            while (m) {
+              const int bb = __ffs(m) - 1;
+              m &= m - 1;
+              const int L2 = g.item_lhs[(w << 5) + bb];
+              if ((bset[L2 >> 5] >> (L2 & 31)) & 1u) add |= 1u << bb;
+            }
+            const uint32_t s = shr1_word(Gk, w, W);
+            if (gap) add |= g.next_any[w] & s;
+            if (self_si >= 0) add |= a.expn[(size_t)self_si * W + w] & s;
+            add &= bits[w];
+            const uint32_t old = Gk[w];
+            if ((old | add) != old) {
+              Gk[w] = old | add;
+              ch = true;
+            }
+          }
+          if (!__any_sync(0xffffffffu, ch)) break;
+          changed = true;
+          if (lane == 0) a.gnz[k] = 1;
+        }
+      }
       if (changed && lane == 0) s_flag = 1;
       __syncthreads();
       const int more = s_flag;
