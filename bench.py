@@ -15,6 +15,7 @@ import argparse
 import json
 import os
 import subprocess
+import tempfile
 import sys
 import time
 
@@ -62,10 +63,12 @@ class Clocks:
     def __init__(self, index):
         self.index = index
         self.proc = None
-        self.path = os.path.join(ROOT, 'gpurun_out', 'bench_clocks.csv')
+        # the raw samples go to EPIC_CLOCKS_CSV when set, else to a temporary file
+        self.path = os.environ.get('EPIC_CLOCKS_CSV') or os.path.join(
+            tempfile.gettempdir(), 'epic_bench_clocks_%d.csv' % os.getpid())
 
     def __enter__(self):
-        os.makedirs(os.path.dirname(self.path), exist_ok=True)
+        os.makedirs(os.path.dirname(os.path.abspath(self.path)), exist_ok=True)
         q = ('index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,'
              'clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,'
              'clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap')
