@@ -20,6 +20,7 @@ constexpr int kMaxFW = 512;
 
 class CoverCols {
  public:
+  static constexpr bool kRecord = false;
   const DevGrammar& g;
   Workspace ws;
   WsDims dims;

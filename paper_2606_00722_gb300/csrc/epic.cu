@@ -792,7 +792,11 @@ epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const in
     int wpc = kWarpsPerCta;
     size_t per = smem_per_warp(sp.nmax, rmax, dg.W, dg.VW);
     if (sm) wpc = (int)std::min<size_t>(kWarpsPerCta, smem_cap / per);
-    if (sm && wpc >= 1) {
+    bool block_walk = false;
+    if (const char* e = getenv("EPIC_FORWARD_BLOCK")) block_walk = atoi(e) != 0;
+    if (block_walk) {
+      k_forward_block<<<B, kThreads, 0, st>>>(dg, t->d_table, t->vocab, d_x, B, n, sp, t->d_stats);
+    } else if (sm && wpc >= 1) {
       size_t dyn = per * wpc;
       cudaFuncSetAttribute(k_forward<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
       k_forward<true><<<(B + wpc - 1) / wpc, 32 * wpc, dyn, st>>>(dg, t->d_table, t->vocab, d_x, B, n, sp, rmax,

@@ -40,6 +40,9 @@ struct SeqArena {
   int32_t* eidx;       // [nmax (nmax + 1) / 2] entry of (column j, origin o <= j), -1: none
   uint8_t* gnz;        // [emax] the entry has a good item
   int32_t* cursor;     // [2 (nmax + 1)] scratch of the good pass
+  int32_t* key_q;      // [kMaxQ] scratch of the block forward walk
+  uint32_t* bexpn;     // [nmax][W]
+  uint32_t* bnew;      // [nmax][VW]
 };
 
 struct SeqPack {
@@ -55,7 +58,8 @@ struct SeqPack {
            + r(nm) + 2 * r((size_t)edge_cap * 4) + r((size_t)edge_cap * 32) + 3 * r((size_t)n * 4) +
            r((size_t)emax * VW * 4) + r(32)                                                 // SeqRec
            + r((size_t)emax * W * 4) + r(nm * 4) + 3 * r((nm + 1) * 4) + r((size_t)edge_cap * 4) +
-           r((size_t)emax * 4) + r(nm * W * 4) + r(nm * (nm + 1) / 2 * 4) + r((size_t)emax) + r(2 * (nm + 1) * 4);
+           r((size_t)emax * 4) + r(nm * W * 4) + r(nm * (nm + 1) / 2 * 4) + r((size_t)emax) + r(2 * (nm + 1) * 4) + r(kMaxQ * 4) +
+           r(nm * W * 4) + r(nm * VW * 4);
   }
   __device__ SeqArena carve(long long b) const {
     SeqArena a;
@@ -103,6 +107,9 @@ struct SeqPack {
     a.eidx = (int32_t*)take(nm * (nm + 1) / 2 * 4);
     a.gnz = (uint8_t*)take((size_t)emax);
     a.cursor = (int32_t*)take(2 * (nm + 1) * 4);
+    a.key_q = (int32_t*)take(kMaxQ * 4);
+    a.bexpn = (uint32_t*)take(nm * W * 4);
+    a.bnew = (uint32_t*)take(nm * VW * 4);
     return a;
   }
 };
@@ -164,6 +171,71 @@ __global__ void __launch_bounds__(32 * kWarpsPerCta) k_forward(DevGrammar g, con
     rec.meta[M_NENT] = (int)walk.nent;
     atomicAdd(&stats[4], (unsigned long long)walk.ncols);  // columns and entries of the forward charts
     atomicAdd(&stats[5], (unsigned long long)walk.nent);
+  }
+}
+
+// The same forward charts with a whole CTA per sequence: the block walk
+// spreads each closure round's dirty origins and completion pairs over the
+// warps (for long sequences of wide grammars, where one warp's walk is a long
+// serial chain).  Selected with EPIC_FORWARD_BLOCK=1.
+__global__ void __launch_bounds__(kThreads) k_forward_block(DevGrammar g, const LexEntry* __restrict__ table,
+                                                            int vocab, const int32_t* __restrict__ x, int B, int n,
+                                                            SeqPack sp, unsigned long long* stats) {
+  __shared__ WalkShared sh;
+  for (long long b = blockIdx.x; b < B; b += gridDim.x) {
+    SeqArena a = sp.carve(b);
+    // the walk expects a zeroed stage and completion record
+    for (size_t w = threadIdx.x; w < (size_t)sp.nmax * g.W; w += blockDim.x) a.ws.stage[w] = 0;
+    for (size_t w = threadIdx.x; w < (size_t)sp.nmax * g.VW; w += blockDim.x) a.ws.bdone[w] = 0;
+    for (int p = threadIdx.x; p < n; p += blockDim.x) {
+      a.rec.gap_col[p] = -1;
+      a.rec.pre_col[p] = -1;
+      a.rec.post_col[p] = -1;
+    }
+    __syncthreads();
+    Workspace ws;
+    ws.stage = a.ws.stage;
+    ws.bdone = a.ws.bdone;
+    ws.col_off = a.ws.col_off;
+    ws.org = a.ws.org;
+    ws.bits = a.ws.bits;
+    ws.cov = nullptr;
+    WalkScratch sc;
+    sc.g_src = a.ws.g_src;
+    sc.g_end = a.ws.g_end;
+    sc.g_len = a.ws.g_len;
+    sc.g_tail = (uint8_t*)a.ws.g_tail;  // [kMaxQ][16] bytes
+    sc.g_lbl = a.ws.g_lbl;
+    sc.g_last = a.ws.g_last;
+    sc.f_q = a.ws.f_q;
+    sc.f_c = a.ws.f_c;
+    sc.key_q = a.key_q;
+    sc.expn = a.bexpn;
+    sc.bnew = a.bnew;
+    const BlockRec br{a.rec.col_gap, a.rec.e_dst,   a.rec.e_src,   a.rec.e_lbl,    a.rec.cnt,
+                      a.ws.esum,     a.rec.gap_col, a.rec.pre_col, a.rec.post_col, a.rec.edge_cap};
+    WsDims d;
+    d.nmax = sp.nmax;
+    d.emax = sp.emax;
+    EarleyColsT<true> cols(g, table, ws, sc, d, sh);
+    cols.rec = &br;
+    Walk<EarleyColsT<true>> walk(cols, g, table, sc, sh, vocab);
+    walk.rec = &br;
+    Subst none{nullptr, nullptr, 0};
+    const int r = walk.run(x + b * n, n, none);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int32_t* meta = a.rec.meta;
+      meta[M_NCOLS] = sh.ncols;
+      meta[M_NEDGES] = sh.nedges;
+      meta[M_START] = sh.start_col;
+      meta[M_ACCEPT] = sh.accept_col;
+      meta[M_STATUS] = r == 1 ? 1 : (r == 0 ? 0 : -1);
+      meta[M_NENT] = (int)sh.nent;
+      atomicAdd(&stats[4], (unsigned long long)sh.ncols);
+      atomicAdd(&stats[5], (unsigned long long)sh.nent);
+    }
+    __syncthreads();
   }
 }
 

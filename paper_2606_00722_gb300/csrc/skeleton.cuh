@@ -16,11 +16,13 @@ struct Walk {
   WalkScratch sc;
   WalkShared& sh;
   int vocab;
+  const BlockRec* rec = nullptr;  // recording walks: positions' columns
 
   __device__ Walk(Cols& c, const DevGrammar& g_, const LexEntry* t, WalkScratch s, WalkShared& shared, int v)
       : cols(c), g(g_), table(t), sc(s), sh(shared), vocab(v) {}
 
   __device__ void label_set(const uint32_t* lbl8) {
+    if (Cols::kRecord && threadIdx.x < 8) sh.lbl8[threadIdx.x] = lbl8[threadIdx.x];
     for (int w = threadIdx.x; w < g.W; w += blockDim.x) {
       uint32_t acc = 0;
       for (int lw = 0; lw < 8; ++lw) {
@@ -37,6 +39,7 @@ struct Walk {
     __syncthreads();
   }
   __device__ void label_one(int a) {
+    if (Cols::kRecord && threadIdx.x < 8) sh.lbl8[threadIdx.x] = (threadIdx.x == (a >> 5)) ? (1u << (a & 31)) : 0u;
     for (int w = threadIdx.x; w < g.W; w += blockDim.x) sh.lbl[w] = g.exp_term[(size_t)a * g.W + w];
     __syncthreads();
   }
@@ -206,6 +209,11 @@ struct Walk {
     return c;
   }
 
+  // positions [lo, hi) of a recording walk -> column c
+  __device__ void rec_range(int32_t* arr, int lo, int hi, int c) {
+    for (int p = lo + threadIdx.x; p < hi; p += blockDim.x) arr[p] = c;
+  }
+
   __device__ int run_inner(const int32_t* x, int n, Subst s) {
     if (n == 0) {
       int c = seed_column(false);
@@ -213,11 +221,13 @@ struct Walk {
       cols.close_column(c, false);
       cols.finish_column(c);
       if (sh.status != kWalkOk) return -1;
+      if (threadIdx.x == 0) sh.accept_col = c;
       return cols.column_has_accept(c, c) ? 1 : 0;
     }
     int i = 0;
     bool first = true;
     int prev_gap = -1;
+    int span_lo = -1, span_hi = -1;  // the last span (recording walks)
     while (i < n) {
       int t0 = token_at(x, s, i);
       int j = i;
@@ -249,6 +259,10 @@ struct Walk {
         cols.close_column(c, true);
         cols.finish_column(c);
         if (sh.status != kWalkOk) return -1;
+        if (Cols::kRecord) {
+          rec_range(rec->gap_col, i, j, c);
+          if (span_lo >= 0) rec_range(rec->post_col, span_lo, span_hi, c);
+        }
         prev_gap = c;
         if (cols.column_empty(c)) return 0;
       } else {
@@ -264,7 +278,9 @@ struct Walk {
             sc.f_c[0] = c;
             sh.nf = 1;
           }
+          if (Cols::kRecord) rec_range(rec->pre_col, i, j, c);
         } else {
+          if (Cols::kRecord) rec_range(rec->pre_col, i, j, prev_gap);
           for (int q = threadIdx.x; q < g.Q; q += blockDim.x) {
             sc.f_q[q] = q;
             sc.f_c[q] = prev_gap;
@@ -272,6 +288,8 @@ struct Walk {
           if (threadIdx.x == 0) sh.nf = g.Q;
         }
         __syncthreads();
+        span_lo = i;
+        span_hi = j;
         for (int p = i; p < j; ++p) {
           if (sh.nf == 0) break;
           int tok = token_at(x, s, p);
@@ -297,12 +315,15 @@ struct Walk {
           cols.close_column(c, false);
           cols.finish_column(c);
           if (sh.status != kWalkOk) return -1;
+          if (Cols::kRecord) rec_range(rec->post_col, i, j, c);
+          if (threadIdx.x == 0) sh.accept_col = c;
           return cols.column_has_accept(c, sh.start_col) ? 1 : 0;
         }
       }
       first = false;
       i = j;
     }
+    if (threadIdx.x == 0) sh.accept_col = prev_gap;
     return cols.column_has_accept(prev_gap, sh.start_col) ? 1 : 0;
   }
 };

@@ -75,6 +75,8 @@ struct WalkShared {
   int32_t changed;
   int32_t nf, ng, nt;
   int32_t start_col, accept_col;
+  int32_t nedges;    // edges recorded so far (recording walks)
+  uint32_t lbl8[8];  // terminal set of the arrivals being made
   int32_t scratch_i[4];
 };
 
@@ -171,8 +173,29 @@ __device__ __forceinline__ bool warp_scan_into(uint32_t* dst, const uint32_t* in
   return __any_sync(0xffffffffu, nz);
 }
 
+// What a recording walk (a sequence's forward chart, for checks by region)
+// writes besides the chart: the graph's edges in target order with their
+// terminal sets (all zero: epsilon), gap flags, each entry's completed
+// nonterminals and folded summaries (bit B mod 32 of a waited-on nonterminal,
+// bit a mod 32 of an expected terminal), and the column before, at and after
+// each position's segment.
+struct BlockRec {
+  uint8_t* col_gap;   // [nmax]
+  int32_t* e_dst;     // [edge_cap]
+  int32_t* e_src;     // [edge_cap]
+  uint32_t* e_lbl;    // [edge_cap][8]
+  uint32_t* cnt;      // [emax][VW]
+  uint32_t* esum;     // [emax][2]
+  int32_t* gap_col;   // [n]
+  int32_t* pre_col;   // [n]
+  int32_t* post_col;  // [n]
+  int edge_cap;
+};
+
 // ------------------------------------------------------------ Earley columns
-class EarleyCols {
+// REC = true: a recording walk (BlockRec), compiled out of the others.
+template <bool REC>
+class EarleyColsT {
  public:
   const DevGrammar& g;
   const LexEntry* table;
@@ -181,8 +204,10 @@ class EarleyCols {
   WsDims dims;
   WalkShared& sh;
   int W, VW;
+  static constexpr bool kRecord = REC;
+  const BlockRec* rec = nullptr;  // recording walks only
 
-  __device__ EarleyCols(const DevGrammar& g_, const LexEntry* t, Workspace w, WalkScratch s, WsDims d,
+  __device__ EarleyColsT(const DevGrammar& g_, const LexEntry* t, Workspace w, WalkScratch s, WsDims d,
                     WalkShared& shared)
       : g(g_), table(t), ws(w), sc(s), dims(d), sh(shared), W(g_.W), VW(g_.VW) {}
   __device__ bool column_has_accept(int c, int start_col) { return accepts(c, start_col); }
@@ -195,6 +220,7 @@ class EarleyCols {
       sh.ncols = 0;
       sh.nent = 0;
       sh.status = kWalkOk;
+      sh.nedges = 0;
       ws.col_off[0] = 0;
     }
     clear_bitmap(sh.touched, kMaxCols);
@@ -222,6 +248,16 @@ class EarleyCols {
   // (M == nullptr and shift == false for an epsilon edge).
   __device__ void arrive(int src, const uint32_t* M, bool shift) {
     int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (REC && threadIdx.x == 0) {  // the edge src -> open column
+      if (sh.nedges >= rec->edge_cap) {
+        sh.status = kWalkOverflow;
+      } else {
+        const int e = sh.nedges++;
+        rec->e_dst[e] = sh.ncols;
+        rec->e_src[e] = src;
+        for (int w = 0; w < 8; ++w) rec->e_lbl[(size_t)e * 8 + w] = shift ? sh.lbl8[w] : 0u;
+      }
+    }
     int b = ws.col_off[src], e = ws.col_off[src + 1];
     for (int k = b + warp; k < e; k += kWarps) {
       int o = ws.org[k];
@@ -246,6 +282,7 @@ class EarleyCols {
   // Closure of column c (is_gap: a gap node with a Sigma_lex* self-loop).
   __device__ void close_column(int c, bool gap) {
     int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (REC && threadIdx.x == 0) rec->col_gap[c] = gap ? 1 : 0;
     for (int round = 0;; ++round) {
       if (round >= kMaxRounds) {
         if (threadIdx.x == 0) sh.status = kWalkOverflow;
@@ -427,6 +464,7 @@ class EarleyCols {
         if (lane == 0) ws.org[base + slot] = o;
         uint32_t* dst = ws.bits + (size_t)(base + slot) * W;
         for (int w = lane; w < W; w += 32) dst[w] = row[w];
+        if constexpr (REC) record_entry(row, (long long)base + slot);
       }
       for (int w = lane; w < W; w += 32) row[w] = 0;
       for (int v = lane; v < VW; v += 32) ws.bdone[(size_t)o * VW + v] = 0;
@@ -440,6 +478,48 @@ class EarleyCols {
   }
 
   __device__ bool column_empty(int c) const { return ws.col_off[c + 1] == ws.col_off[c]; }
+
+  // Warp: completed nonterminals and folded summaries of stored entry k.
+  __device__ void record_entry(const uint32_t* row, long long k) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint32_t* nts = sh.wnt[warp];
+    for (int v = lane; v < VW; v += 32) nts[v] = 0;
+    __syncwarp();
+    uint32_t fnt = 0, ft = 0;
+    for (int w = lane; w < W; w += 32) {
+      const uint32_t r = row[w];
+      uint32_t m = r & g.complete[w];
+      while (m) {
+        const int b = __ffs(m) - 1;
+        m &= m - 1;
+        const int B = g.item_lhs[(w << 5) + b];
+        atomicOr(&nts[B >> 5], 1u << (B & 31));
+      }
+      m = r & g.any_nt[w];
+      while (m) {
+        const int b = __ffs(m) - 1;
+        m &= m - 1;
+        fnt |= 1u << ((g.item_next[(w << 5) + b] - g.T) & 31);
+      }
+      m = r & g.any_term[w];
+      while (m) {
+        const int b = __ffs(m) - 1;
+        m &= m - 1;
+        ft |= 1u << (g.item_next[(w << 5) + b] & 31);
+      }
+    }
+    for (int off = 16; off; off >>= 1) {
+      fnt |= __shfl_xor_sync(0xffffffffu, fnt, off);
+      ft |= __shfl_xor_sync(0xffffffffu, ft, off);
+    }
+    __syncwarp();
+    for (int v = lane; v < VW; v += 32) rec->cnt[(size_t)k * VW + v] = nts[v];
+    if (lane == 0) {
+      rec->esum[(size_t)k * 2] = fnt;
+      rec->esum[(size_t)k * 2 + 1] = ft;
+    }
+    __syncwarp();
+  }
 
   // After an aborted walk: return the staging rows of the open column to zero.
   __device__ void cleanup() {
@@ -471,5 +551,7 @@ class EarleyCols {
   }
 
 };
+
+using EarleyCols = EarleyColsT<false>;
 
 }  // namespace epic
