@@ -136,6 +136,14 @@ epic_status epic_lexer_table_copy(const epic_lexer_table* t, int32_t first_token
  * EPIC_ERR_INVALID_ARG for sizes < 0 or NULL pointers with non-empty sizes.
  * Device-side: an unmasked position or an out-of-range token id yields 0 for
  * that check and counts in stats.bad_inputs.  Asynchronous.
+ * Two strategies give identical results: one warp per check walking the
+ * whole graph of x (+) (pos, tok); or, when item sets exceed 32 words or the
+ * batch has more checks than resident walks, one forward chart of x per
+ * sequence (with its graph and good-item masks) and one warp per check
+ * walking only the candidate's region (stats.region_checks counts these).
+ * The library's device workspaces grow on demand (the per-sequence charts
+ * up to EPIC_SEQ_WORKSPACE_MB, default 80 GiB); a failed allocation returns
+ * EPIC_ERR_OOM.  A sequence whose chart does not fit walks its checks whole.
  */
 epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t,
                                 const int32_t* d_x, int32_t B, int32_t n, const int32_t* d_pos,
