@@ -12,8 +12,7 @@
 
 #include "../../include/epic.h"
 #include "grammar.h"
-#include "skeleton.cuh"
-#include "warpwalk.cuh"
+#include "launch.h"
 
 using namespace epic;
 
@@ -64,208 +63,6 @@ __global__ void k_lex_table(const int32_t* __restrict__ tok_off, const uint8_t* 
   table[idx] = e;
 }
 
-struct WsPack {
-  char* base;
-  size_t per_cta;
-  WsDims dims;
-  int W, VW, FW;
-  __device__ void carve(int cta, Workspace& ws, WalkScratch& sc) const {
-    char* p = base + per_cta * (size_t)cta;
-    auto take = [&](size_t bytes) {
-      char* r = p;
-      p += (bytes + 255) & ~(size_t)255;
-      return r;
-    };
-    int nm = dims.nmax;
-    ws.stage = (uint32_t*)take((size_t)nm * W * 4);
-    ws.bdone = (uint32_t*)take((size_t)nm * VW * 4);
-    ws.col_off = (int32_t*)take((size_t)(nm + 1) * 4);
-    ws.cov = (uint32_t*)take((size_t)nm * FW * 4);
-    sc.g_src = (int32_t*)take(kMaxQ * 4);
-    sc.g_end = (int32_t*)take(kMaxQ * 4);
-    sc.g_len = (int32_t*)take(kMaxQ * 4);
-    sc.g_last = (int32_t*)take(kMaxQ * 4);
-    sc.f_q = (int32_t*)take(kMaxQ * 4);
-    sc.f_c = (int32_t*)take(kMaxQ * 4);
-    sc.key_q = (int32_t*)take(kMaxQ * 4);
-    sc.g_tail = (uint8_t*)take(kMaxQ * 16);
-    sc.g_lbl = (uint32_t*)take(kMaxQ * 8 * 4);
-    sc.expn = (uint32_t*)take((size_t)nm * W * 4);
-    sc.bnew = (uint32_t*)take((size_t)nm * VW * 4);
-    ws.org = (int32_t*)take((size_t)dims.emax * 4);
-    ws.bits = (uint32_t*)take((size_t)dims.emax * W * 4);
-  }
-};
-
-static size_t ws_bytes_per_cta(const WsDims& d, int W, int VW, int FW) {
-  auto r = [](size_t b) { return (b + 255) & ~(size_t)255; };
-  size_t nm = d.nmax;
-  return r(nm * W * 4) + r(nm * VW * 4) + r((nm + 1) * 4) + r(nm * FW * 4) + 7 * r(kMaxQ * 4) +
-         r(kMaxQ * 16) + r(kMaxQ * 32) + r(nm * W * 4) + r(nm * VW * 4) + r((size_t)d.emax * 4) +
-         r((size_t)d.emax * W * 4);
-}
-
-enum StatIdx { S_CHECKS, S_VALID, S_OVERFLOW, S_BAD, S_COLUMNS, S_ENTRIES, S_COVER, S_EXACT, S_SELECTED, S_N };
-
-// shared-memory staging of one warp: rows, completed-NT sets, slot origins,
-// origin slots (16-byte multiple)
-__host__ __device__ inline size_t smem_per_warp(int nmax, int rmax, int W, int VW) {
-  size_t b = (size_t)rmax * W * 4 + (size_t)rmax * VW * 4 + (size_t)rmax * 4 + (size_t)rmax * 8 + (size_t)nmax * 2;
-  return (b + 15) & ~(size_t)15;
-}
-
-struct WPack {
-  char* base;
-  size_t per_warp;
-  int nmax;
-  long long emax;
-  int W, VW;
-  __device__ WWs carve(long long warp) const {
-    WWs ws;
-    char* p = base + per_warp * (size_t)warp;
-    auto take = [&](size_t bytes) {
-      char* r = p;
-      p += (bytes + 255) & ~(size_t)255;
-      return r;
-    };
-    ws.stage = (uint32_t*)take((size_t)nmax * W * 4);
-    ws.bdone = (uint32_t*)take((size_t)nmax * VW * 4);
-    ws.col_off = (int32_t*)take((size_t)(nmax + 1) * 4);
-    ws.f_q = (int32_t*)take(kWMaxQ * 4);
-    ws.f_c = (int32_t*)take(kWMaxQ * 4);
-    ws.g_src = (int32_t*)take(kWMaxQ * 4);
-    ws.g_end = (int32_t*)take(kWMaxQ * 4);
-    ws.g_len = (int32_t*)take(kWMaxQ * 4);
-    ws.g_last = (int32_t*)take(kWMaxQ * 4);
-    ws.g_tail = (uint32_t*)take(kWMaxQ * 16);
-    ws.g_lbl = (uint32_t*)take(kWMaxQ * 32);
-    ws.ssum = (uint32_t*)take((size_t)nmax * 8);
-    ws.org = (int32_t*)take((size_t)emax * 4);
-    ws.esum = (uint32_t*)take((size_t)emax * 8);
-    ws.bits = (uint32_t*)take((size_t)emax * W * 4);
-    return ws;
-  }
-};
-
-static size_t wbytes_per_warp(int nmax, long long emax, int W, int VW) {
-  auto r = [](size_t b) { return (b + 255) & ~(size_t)255; };
-  return r((size_t)nmax * W * 4) + r((size_t)nmax * VW * 4) + r((size_t)(nmax + 1) * 4) + 6 * r(kWMaxQ * 4) +
-         r(kWMaxQ * 16) + r(kWMaxQ * 32) + r((size_t)nmax * 8) + r((size_t)emax * 4) + r((size_t)emax * 8) +
-         r((size_t)emax * W * 4);
-}
-
-// K2-K4 (warp form): one warp per validity check; warps pull checks from a
-// counter.  Each check walks the lexeme graph of x (+) (pos, tok) and runs
-// bit-parallel Earley recognition over it.
-// Bytes of the grammar tables the warp walk reads, staged in shared memory
-// (16-byte aligned pieces).
-__host__ __device__ inline size_t gtab_bytes(int T, int V, int W, int D, int Q) {
-  auto r = [](size_t b) { return (b + 15) & ~(size_t)15; };
-  return r((size_t)T * W * 4) + 2 * r((size_t)V * W * 4) + r((size_t)V * W * 4) + 5 * r((size_t)W * 4) +
-         2 * r((size_t)D * 2) + r((size_t)Q * 2) + r((size_t)Q) + r((size_t)T);
-}
-
-// Copy the walk's grammar tables into shared memory and point `out` at them.
-__device__ void stage_grammar(const DevGrammar& g, unsigned char* smem, DevGrammar& out) {
-  out = g;
-  unsigned char* p = smem;
-  auto put = [&](const void* src, size_t bytes) -> void* {
-    void* dst = p;
-    const uint32_t* s4 = (const uint32_t*)src;
-    uint32_t* d4 = (uint32_t*)dst;
-    size_t n4 = bytes / 4;
-    for (size_t i = threadIdx.x; i < n4; i += blockDim.x) d4[i] = s4[i];
-    for (size_t i = n4 * 4 + threadIdx.x; i < bytes; i += blockDim.x)
-      ((unsigned char*)dst)[i] = ((const unsigned char*)src)[i];
-    p += (bytes + 15) & ~(size_t)15;
-    return dst;
-  };
-  out.exp_term = (const uint32_t*)put(g.exp_term, (size_t)g.T * g.W * 4);
-  out.exp_nt = (const uint32_t*)put(g.exp_nt, (size_t)g.V * g.W * 4);
-  out.pred = (const uint32_t*)put(g.pred, (size_t)g.V * g.W * 4);
-  out.gap_pred = (const uint32_t*)put(g.gap_pred, (size_t)g.V * g.W * 4);
-  out.any_nt = (const uint32_t*)put(g.any_nt, (size_t)g.W * 4);
-  out.any_term = (const uint32_t*)put(g.any_term, (size_t)g.W * 4);
-  out.next_any = (const uint32_t*)put(g.next_any, (size_t)g.W * 4);
-  out.nullable_next = (const uint32_t*)put(g.nullable_next, (size_t)g.W * 4);
-  out.complete = (const uint32_t*)put(g.complete, (size_t)g.W * 4);
-  out.item_next = (const int16_t*)put(g.item_next, (size_t)g.D * 2);
-  out.item_lhs = (const int16_t*)put(g.item_lhs, (size_t)g.D * 2);
-  out.dfa_accept = (const int16_t*)put(g.dfa_accept, (size_t)g.Q * 2);
-  out.dfa_ext = (const uint8_t*)put(g.dfa_ext, (size_t)g.Q);
-  out.skip = (const uint8_t*)put(g.skip, (size_t)g.T);
-  __syncthreads();
-}
-
-template <bool SM>
-__global__ void __launch_bounds__(32 * kWarpsPerCta) k_validate_warp(
-    DevGrammar g, const LexEntry* __restrict__ table, int vocab, const int32_t* __restrict__ x, int n,
-    const int32_t* __restrict__ pos, int k, const int32_t* __restrict__ cand, int K, long long total,
-    uint8_t* __restrict__ valid, WPack wp, int rmax, int gtab_smem, unsigned long long* counter,
-    unsigned long long* stats) {
-  __shared__ WSh shm[kWarpsPerCta];
-  extern __shared__ __align__(16) unsigned char dyn[];
-  int warp = threadIdx.x >> 5;
-  WSh& sh = shm[warp];
-  for (int w = threadIdx.x & 31; w < kWCols / 32; w += 32) {
-    sh.touched[w] = 0;
-    sh.dirty[w] = 0;
-  }
-  for (int v = threadIdx.x & 31; v < kWMaxVW; v += 32) {
-    sh.vset[v] = 0;
-    sh.vdone[v] = 0;
-  }
-  __syncwarp();
-  // the grammar tables in shared memory when they fit (gtab > 0)
-  DevGrammar gs = g;
-  size_t gt = 0;
-  if constexpr (SM) {
-    if (gtab_smem) {
-      stage_grammar(g, dyn, gs);
-      gt = gtab_bytes(g.T, g.V, g.W, g.D, g.Q);
-    }
-  }
-  WarpWalker<SM> walk(gs, table, wp.carve((long long)blockIdx.x * (blockDim.x >> 5) + warp), sh, wp.nmax, wp.emax,
-                      vocab);
-  if constexpr (SM) {
-    size_t per = smem_per_warp(wp.nmax, rmax, g.W, g.VW);
-    unsigned char* base = dyn + gt + per * warp;
-    uint32_t* rows = (uint32_t*)base;
-    uint32_t* bd = rows + (size_t)rmax * g.W;
-    int32_t* sorg = (int32_t*)(bd + (size_t)rmax * g.VW);
-    uint32_t* ssum = (uint32_t*)(sorg + rmax);
-    int16_t* so = (int16_t*)(ssum + 2 * rmax);
-    walk.set_smem(rows, bd, so, sorg, ssum, rmax);
-  }
-  unsigned long long n_checks = 0, n_valid = 0, n_ovf = 0, n_bad = 0, n_cols = 0, n_ent = 0;
-  for (;;) {
-    long long jb = 0;
-    if ((threadIdx.x & 31) == 0) jb = (long long)atomicAdd(counter, 1ull);
-    jb = __shfl_sync(0xffffffffu, jb, 0);
-    if (jb >= total) break;
-    long long b = jb / ((long long)k * K);
-    long long j = (jb / K) % k;
-    int r = walk.run(x + b * n, n, pos[b * k + j], cand[jb]);
-    if ((threadIdx.x & 31) == 0) valid[jb] = r == 1 ? 1 : (r == -1 ? 2 : 0);
-    ++n_checks;
-    n_valid += r == 1;
-    n_ovf += r == -1;
-    n_bad += r == -2;
-    n_cols += walk.ncols;
-    n_ent += walk.nent;
-  }
-  if ((threadIdx.x & 31) == 0 && n_checks) {
-    atomicAdd(&stats[S_CHECKS], n_checks);
-    atomicAdd(&stats[S_VALID], n_valid);
-    atomicAdd(&stats[S_OVERFLOW], n_ovf);
-    atomicAdd(&stats[S_BAD], n_bad);
-    atomicAdd(&stats[S_COLUMNS], n_cols);
-    atomicAdd(&stats[S_ENTRIES], n_ent);
-  }
-}
-
-#include "region.cuh"
-
 // Per proposed position: the highest-confidence candidate with valid bit 1.
 __global__ void k_pick(const int32_t* __restrict__ cand, const float* __restrict__ conf,
                        const uint8_t* __restrict__ valid, int B, int k, int K, int32_t* __restrict__ tok,
@@ -285,265 +82,6 @@ __global__ void k_pick(const int32_t* __restrict__ cand, const float* __restrict
   }
   tok[i] = best < 0 ? -1 : cand[i * K + best];
   out_conf[i] = best < 0 ? 0.f : bc;
-}
-
-// Alg. 4 per sequence: one CTA runs RelaxedSelect / ExactShrink with an
-// explicit stack; thread 0 drives the recursion, the whole CTA runs each
-// cover test (CoverCols walk) and exact joint check (EarleyCols walk).
-constexpr int kMaxSel = 64;
-
-struct SelFrame {
-  int8_t kind;  // 0 root, 1 relaxed, 2 shrink
-  int8_t pc;
-  unsigned long long base, set, a, b;
-};
-
-// Alg. 4 always starts with the cover test of x (+) C and, when that passes,
-// continues with the exact test of the same x (+) C.  Both are run here at
-// once, one CTA each per sequence, before the recursion; k_select reuses the
-// two answers when it asks for exactly these tests.  spec[b] = {cover,
-// exact}: 1 pass, 0 fail, -1 not available (overflow / bad input).
-__global__ void __launch_bounds__(kThreads) k_select_spec(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
-                                                          const int32_t* __restrict__ x, int B, int n,
-                                                          const int32_t* __restrict__ pos, int k,
-                                                          const int32_t* __restrict__ tok, int8_t* __restrict__ spec,
-                                                          WsPack wsp) {
-  __shared__ WalkShared sh;
-  __shared__ int s_pos[kMaxSel], s_tok[kMaxSel];
-  __shared__ int ns;
-  Workspace ws;
-  WalkScratch sc;
-  wsp.carve(blockIdx.x, ws, sc);
-  for (int job = blockIdx.x; job < 2 * B; job += gridDim.x) {
-    int b = job >> 1;
-    bool exact = job & 1;
-    if (threadIdx.x == 0) {
-      int m = 0;
-      for (int j = 0; j < k; ++j) {
-        int t = tok[(long long)b * k + j];
-        if (t < 0) continue;
-        s_pos[m] = pos[(long long)b * k + j];
-        s_tok[m] = t;
-        ++m;
-      }
-      ns = m;
-    }
-    __syncthreads();
-    int r = -1;
-    if (ns >= 2) {  // a set of at most one candidate is never tested
-      Subst s{s_pos, s_tok, ns};
-      if (exact) {
-        EarleyCols cols(g, table, ws, sc, wsp.dims, sh);
-        Walk<EarleyCols> w(cols, g, table, sc, sh, vocab);
-        r = w.run(x + (long long)b * n, n, s);
-      } else {
-        CoverCols cols(g, ws, wsp.dims, sh);
-        Walk<CoverCols> w(cols, g, table, sc, sh, vocab);
-        r = w.run(x + (long long)b * n, n, s);
-      }
-    }
-    if (threadIdx.x == 0) spec[2 * b + (exact ? 1 : 0)] = (int8_t)(r == 1 ? 1 : (r == 0 ? 0 : -1));
-    __syncthreads();
-  }
-}
-
-__global__ void __launch_bounds__(kThreads) k_select(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
-                                                     const int32_t* __restrict__ x, int B, int n,
-                                                     const int32_t* __restrict__ pos, int k,
-                                                     const int32_t* __restrict__ tok, const float* __restrict__ conf,
-                                                     uint8_t* __restrict__ selected, WsPack wsp,
-                                                     const int8_t* __restrict__ spec, unsigned long long* stats) {
-  __shared__ WalkShared sh;
-  __shared__ int c_slot[kMaxSel], c_pos[kMaxSel], c_tok[kMaxSel];
-  __shared__ int s_pos[kMaxSel], s_tok[kMaxSel];
-  __shared__ SelFrame stack[2 * kMaxSel + 8];
-  __shared__ int sp, nc, action, result, bad, overflow;
-  __shared__ unsigned long long ret, final_set;
-  Workspace ws;
-  WalkScratch sc;
-  wsp.carve(blockIdx.x, ws, sc);
-  EarleyCols ecols(g, table, ws, sc, wsp.dims, sh);
-  CoverCols ccols(g, ws, wsp.dims, sh);
-  Walk<EarleyCols> exact(ecols, g, table, sc, sh, vocab);
-  Walk<CoverCols> cover(ccols, g, table, sc, sh, vocab);
-  for (int b = blockIdx.x; b < B; b += gridDim.x) {
-    const int32_t* xb = x + (long long)b * n;
-    if (threadIdx.x == 0) {
-      // C: proposed (position, token) pairs, by descending confidence then
-      // ascending position (insertion sort; k <= 64)
-      int m = 0;
-      bad = 0;
-      overflow = 0;
-      for (int j = 0; j < k; ++j) {
-        int t = tok[(long long)b * k + j];
-        if (t < 0) continue;
-        float cf = conf[(long long)b * k + j];
-        if (cf != cf) bad = 1;
-        int p = pos[(long long)b * k + j];
-        int i = m++;
-        while (i > 0) {
-          float cp = conf[(long long)b * k + c_slot[i - 1]];
-          if (cp > cf || (cp == cf && c_pos[i - 1] < p)) break;
-          c_slot[i] = c_slot[i - 1];
-          c_pos[i] = c_pos[i - 1];
-          c_tok[i] = c_tok[i - 1];
-          --i;
-        }
-        c_slot[i] = j;
-        c_pos[i] = p;
-        c_tok[i] = t;
-      }
-      nc = m;
-      sp = 0;
-      stack[0] = SelFrame{0, 0, 0ull, nc == 64 ? ~0ull : ((1ull << nc) - 1), 0ull, 0ull};
-      sp = 1;
-      final_set = 0;
-      if (bad) sp = 0;
-    }
-    __syncthreads();
-    for (;;) {
-      // thread 0 advances the recursion until it needs a test or finishes
-      if (threadIdx.x == 0) {
-        action = 0;
-        while (sp > 0 && action == 0) {
-          if (sp >= 2 * kMaxSel + 6) {  // recursion deeper than Alg. 4 can go
-            overflow = 1;
-            sp = 0;
-            break;
-          }
-          SelFrame& f = stack[sp - 1];
-          unsigned long long set = f.set;
-          // split in confidence order: first ceil(|set|/2) members
-          auto halves = [&](unsigned long long s, unsigned long long& L, unsigned long long& R) {
-            int cnt = __popcll(s), h = (cnt + 1) / 2;
-            L = 0;
-            unsigned long long r = s;
-            for (int i = 0; i < h; ++i) {
-              unsigned long long lo = r & (~r + 1);
-              L |= lo;
-              r &= r - 1;
-            }
-            R = s & ~L;
-          };
-          if (f.kind == 0) {
-            if (f.pc == 0) {
-              f.pc = 1;
-              stack[sp++] = SelFrame{1, 0, 0ull, set, 0ull, 0ull};
-            } else if (f.pc == 1) {
-              f.pc = 2;
-              stack[sp++] = SelFrame{2, 0, 0ull, ret, 0ull, 0ull};
-            } else {
-              final_set = ret;
-              --sp;
-            }
-          } else if (f.kind == 1) {  // RelaxedSelect(x (+) base, set)
-            if (f.pc == 0) {
-              if (__popcll(set) <= 1) {
-                ret = 0;
-                --sp;
-              } else {
-                f.pc = 1;
-                action = 1;  // cover test of base | set
-                f.a = f.base | set;
-              }
-            } else if (f.pc == 1) {
-              if (result == 1) {
-                ret = set;
-                --sp;
-              } else {
-                unsigned long long L, R;
-                halves(set, L, R);
-                f.a = R;
-                f.pc = 2;
-                stack[sp++] = SelFrame{1, 0, f.base, L, 0ull, 0ull};
-              }
-            } else if (f.pc == 2) {
-              f.b = ret;
-              f.pc = 3;
-              unsigned long long R = f.a;
-              stack[sp++] = SelFrame{1, 0, f.base | ret, R, 0ull, 0ull};
-            } else {
-              ret = f.b | ret;
-              --sp;
-            }
-          } else {  // ExactShrink(x (+) base, set)
-            if (f.pc == 0) {
-              if (__popcll(set) <= 1) {
-                ret = 0;
-                --sp;
-              } else {
-                f.pc = 1;
-                action = 2;  // exact joint check of base | set
-                f.a = f.base | set;
-              }
-            } else if (f.pc == 1) {
-              if (result == 1) {
-                ret = set;
-                --sp;
-              } else {
-                unsigned long long L, R;
-                halves(set, L, R);
-                f.a = R;
-                f.pc = 2;
-                stack[sp++] = SelFrame{2, 0, f.base, L, 0ull, 0ull};
-              }
-            } else if (f.pc == 2) {
-              f.b = ret;  // B'_L
-              f.pc = 3;
-              stack[sp++] = SelFrame{1, 0, f.base | ret, f.a, 0ull, 0ull};
-            } else if (f.pc == 3) {
-              f.pc = 4;
-              stack[sp++] = SelFrame{2, 0, f.base | f.b, ret, 0ull, 0ull};
-            } else {
-              ret = f.b | ret;
-              --sp;
-            }
-          }
-        }
-        if (action != 0) {
-          unsigned long long m = stack[sp - 1].a;
-          int ns = 0;
-          for (int i = 0; i < nc; ++i)
-            if ((m >> i) & 1ull) {
-              s_pos[ns] = c_pos[i];
-              s_tok[ns] = c_tok[i];
-              ++ns;
-            }
-          result = ns;  // substitution count for the test
-        }
-      }
-      __syncthreads();
-      int act = action;
-      if (act == 0) break;
-      Subst s{s_pos, s_tok, result};
-      // the test of the whole candidate set was run ahead (k_select_spec)
-      unsigned long long full = nc == 64 ? ~0ull : ((1ull << nc) - 1);
-      int cached = (spec && stack[sp - 1].a == full) ? spec[2 * b + (act == 1 ? 0 : 1)] : -1;
-      __syncthreads();
-      int r = cached >= 0 ? cached : ((act == 1) ? cover.run(xb, n, s) : exact.run(xb, n, s));
-      if (threadIdx.x == 0) {
-        if (r < 0) {
-          overflow |= (r == -1);
-          bad |= (r == -2);
-          sp = 0;
-        }
-        result = r == 1 ? 1 : 0;
-        atomicAdd(&stats[act == 1 ? S_COVER : S_EXACT], 1ull);
-      }
-      __syncthreads();
-    }
-    if (threadIdx.x == 0) {
-      for (int j = 0; j < k; ++j) selected[(long long)b * k + j] = overflow ? 2 : 0;
-      if (!overflow && !bad) {
-        for (int i = 0; i < nc; ++i)
-          if ((final_set >> i) & 1ull) selected[(long long)b * k + c_slot[i]] = 1;
-        atomicAdd(&stats[S_SELECTED], (unsigned long long)__popcll(final_set));
-      }
-      if (bad) atomicAdd(&stats[S_BAD], 1ull);
-      if (overflow) atomicAdd(&stats[S_OVERFLOW], 1ull);
-    }
-    __syncthreads();
-  }
 }
 
 __global__ void k_commit(int32_t* __restrict__ x, int B, int n, const int32_t* __restrict__ pos, int k,
@@ -795,19 +333,18 @@ epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const in
     bool block_walk = false;
     if (const char* e = getenv("EPIC_FORWARD_BLOCK")) block_walk = atoi(e) != 0;
     if (block_walk) {
-      k_forward_block<<<B, kThreads, 0, st>>>(dg, t->d_table, t->vocab, d_x, B, n, sp, t->d_stats);
+      launch_forward_block(B, st, dg, t->d_table, t->vocab, d_x, B, n, sp, t->d_stats);
     } else if (sm && wpc >= 1) {
       size_t dyn = per * wpc;
-      cudaFuncSetAttribute(k_forward<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-      k_forward<true><<<(B + wpc - 1) / wpc, 32 * wpc, dyn, st>>>(dg, t->d_table, t->vocab, d_x, B, n, sp, rmax,
-                                                                    t->d_stats);
+      launch_forward(true, (B + wpc - 1) / wpc, 32 * wpc, dyn, st, dg, t->d_table, t->vocab, d_x, B, n, sp, rmax,
+                     t->d_stats);
     } else {
-      k_forward<false><<<(B + kWarpsPerCta - 1) / kWarpsPerCta, 32 * kWarpsPerCta, 0, st>>>(
-          dg, t->d_table, t->vocab, d_x, B, n, sp, 0, t->d_stats);
+      launch_forward(false, (B + kWarpsPerCta - 1) / kWarpsPerCta, 32 * kWarpsPerCta, 0, st, dg, t->d_table,
+                     t->vocab, d_x, B, n, sp, 0, t->d_stats);
     }
   }
   // 2. good masks
-  k_good<<<B, 32 * kGoodWarps, 0, st>>>(dg, B, sp);
+  launch_good(B, st, dg, B, sp);
   t->n_region += total;
   t->n_vkernels += 3;
   // 3. checks
@@ -818,14 +355,13 @@ epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const in
   if (wpc >= 1) {
     int blocks = (int)std::max<long long>(1, warps / wpc);
     size_t dyn = per * wpc;
-    cudaFuncSetAttribute(k_check<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-    k_check<true><<<blocks, 32 * wpc, dyn, st>>>(dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total, d_valid,
-                                                 sp, wp, t->d_regs, rmax, t->d_counter, t->d_stats);
+    launch_check_sm(blocks, 32 * wpc, dyn, st, dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total, d_valid,
+                    sp, wp, t->d_regs, rmax, t->d_counter, t->d_stats);
   } else {
     int per_cta = (int)std::min<long long>(kWarpsPerCta, warps);
     int blocks = (int)std::max<long long>(1, warps / per_cta);
-    k_check<false><<<blocks, 32 * per_cta, 0, st>>>(dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total,
-                                                    d_valid, sp, wp, t->d_regs, 0, t->d_counter, t->d_stats);
+    launch_check_global(blocks, 32 * per_cta, 0, st, dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total,
+                        d_valid, sp, wp, t->d_regs, 0, t->d_counter, t->d_stats);
   }
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
 }
@@ -849,11 +385,10 @@ extern "C" {
 // measurement build only: per-phase cycle counters of the warp walker
 int epic_debug_phase_read(unsigned long long* out16, int reset) {
   if (cudaDeviceSynchronize() != cudaSuccess) return -1;
-  if (cudaMemcpyFromSymbol(out16, g_phase, sizeof(unsigned long long) * 16) != cudaSuccess) return -1;
-  if (reset) {
-    unsigned long long z[16] = {0};
-    cudaMemcpyToSymbol(g_phase, z, sizeof(z));
-  }
+  for (int i = 0; i < 16; ++i) out16[i] = 0;
+  if (phase_read_walk(out16, reset) != 0 || phase_read_forward(out16, reset) != 0 ||
+      phase_read_check_sm(out16, reset) != 0 || phase_read_check_global(out16, reset) != 0)
+    return -1;
   return 0;
 }
 #endif
@@ -1114,13 +649,11 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
     size_t dyn = per * wpc + (gsm ? gt : 0);
     int blocks = (t->wwarps + wpc - 1) / wpc;
     if ((size_t)blocks * wpc > (size_t)t->wwarps) blocks = t->wwarps / wpc;
-    cudaFuncSetAttribute(k_validate_warp<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-    k_validate_warp<true><<<blocks, 32 * wpc, dyn, st>>>(g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K,
-                                                          total, d_valid, wp, rmax, gsm, t->d_counter, t->d_stats);
+    launch_validate_warp(true, blocks, 32 * wpc, dyn, st, g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K,
+                         total, d_valid, wp, rmax, gsm, t->d_counter, t->d_stats);
   } else {
-    k_validate_warp<false><<<t->wwarps / kWarpsPerCta, 32 * kWarpsPerCta, 0, st>>>(
-        g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total, d_valid, wp, 0, 0, t->d_counter,
-        t->d_stats);
+    launch_validate_warp(false, t->wwarps / kWarpsPerCta, 32 * kWarpsPerCta, 0, st, g->dg, t->d_table, t->vocab, d_x,
+                         n, d_pos, k, d_cand, K, total, d_valid, wp, 0, 0, t->d_counter, t->d_stats);
   }
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
 }
@@ -1185,18 +718,16 @@ epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_
     int per_cta = (int)std::min<long long>(wpc, warps);
     int blocks = (int)(warps / per_cta);
     size_t dyn = sper * per_cta;
-    cudaFuncSetAttribute(k_validate_warp<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-    k_validate_warp<true><<<blocks, 32 * per_cta, dyn, st>>>(g->dg, t->d_table, t->vocab, d_x, n, d_pos, k,
-                                                              d_cand, K, total, d_valid, wp, rmax, 0, counter,
-                                                              t->d_stats);
+    launch_validate_warp(true, blocks, 32 * per_cta, dyn, st, g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand,
+                         K, total, d_valid, wp, rmax, 0, counter, t->d_stats);
   } else {
     // the global stage and its completed-NT sets must start at zero
     long long warps = std::min<long long>({total, fit, (long long)sm_count() * 2 * kWarpsPerCta});
     int per_cta = (int)std::min<long long>(kWarpsPerCta, warps);
     int blocks = (int)(warps / per_cta);
     if (cudaMemsetAsync(wp.base, 0, wp.per_warp * (size_t)blocks * per_cta, st) != cudaSuccess) return EPIC_ERR_CUDA;
-    k_validate_warp<false><<<blocks, 32 * per_cta, 0, st>>>(g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand,
-                                                             K, total, d_valid, wp, 0, 0, counter, t->d_stats);
+    launch_validate_warp(false, blocks, 32 * per_cta, 0, st, g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand,
+                         K, total, d_valid, wp, 0, 0, counter, t->d_stats);
   }
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
 }
@@ -1234,11 +765,11 @@ epic_status epic_select_compatible_subset(const epic_grammar* g, const epic_lexe
     t->spec_cap = B;
   }
   t->last = st;
-  k_select_spec<<<std::min(2 * B, t->ctas), kThreads, 0, st>>>(g->dg, t->d_table, t->vocab, d_x, B, n, d_pos, k,
-                                                              d_tok, t->d_spec, pack_of(t));
+  launch_select_spec(std::min(2 * B, t->ctas), st, g->dg, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_tok,
+                     t->d_spec, pack_of(t));
   int ctas = std::min(B, t->ctas);
-  k_select<<<ctas, kThreads, 0, st>>>(g->dg, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_tok, d_conf, d_selected,
-                                      pack_of(t), t->d_spec, t->d_stats);
+  launch_select(ctas, st, g->dg, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_tok, d_conf, d_selected, pack_of(t),
+                t->d_spec, t->d_stats);
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
 }
 

@@ -84,7 +84,7 @@ __device__ __forceinline__ bool bit_get(const uint32_t* m, int i) { return (m[i 
 
 // ------------------------------------------------------------ block helpers
 // Compact the set bits of bitmap[0 .. nbits) into sh.list (ascending).
-__device__ void bitmap_to_list(WalkShared& sh, const uint32_t* bitmap, int nbits) {
+__device__ inline void bitmap_to_list(WalkShared& sh, const uint32_t* bitmap, int nbits) {
   int nw = (nbits + 31) >> 5;
   for (int w = threadIdx.x; w < nw; w += blockDim.x) sh.prefix[w] = __popc(bitmap[w]);
   __syncthreads();
@@ -116,7 +116,7 @@ __device__ __forceinline__ void clear_bitmap(uint32_t* bm, int nbits) {
 
 // Warp: row |= shift(row & M) for a W-word row, until stable; returns true if
 // anything changed.  Item (p, d) is bit i, (p, d+1) is bit i+1.
-__device__ bool warp_advance_closure(uint32_t* row, const uint32_t* M, int W) {
+__device__ inline bool warp_advance_closure(uint32_t* row, const uint32_t* M, int W) {
   int lane = threadIdx.x & 31;
   bool any = false;
   for (int it = 0; it < 64; ++it) {

@@ -108,7 +108,7 @@ __device__ __forceinline__ void expn_of_set(const DevGrammar& g, const uint32_t*
 }
 
 #ifdef EPIC_PHASE_TIMERS
-__device__ unsigned long long g_phase[16];
+static __device__ unsigned long long g_phase[16];  // one per translation unit
 #define PH_BEGIN(v) long long v = clock64()
 #define PH_END(i, v)                                              \
   do {                                                            \

@@ -15,13 +15,18 @@ import subprocess
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SRC = [os.path.join(_HERE, 'csrc', f) for f in ('epic.cu', 'grammar.cpp')]
+# translation units, compiled in parallel and linked into one library
+_SRC = [os.path.join(_HERE, 'csrc', f) for f in
+        ('epic.cu', 'kernels_walk.cu', 'kernels_select.cu', 'region_forward.cu', 'region_good.cu',
+         'region_check_sm.cu', 'region_check_global.cu', 'grammar.cpp')]
 _DEPS = _SRC + [os.path.join(_HERE, 'csrc', f) for f in
-                ('grammar.h', 'device.cuh', 'walk.cuh', 'cover.cuh', 'skeleton.cuh', 'warpwalk.cuh', 'region.cuh')] + \
+                ('grammar.h', 'device.cuh', 'walk.cuh', 'cover.cuh', 'skeleton.cuh', 'warpwalk.cuh', 'packs.cuh',
+                 'seqpack.cuh', 'launch.h', 'region.cuh', 'region_check.cuh')] + \
     [os.path.join(_HERE, '..', 'include', 'epic.h')]
 LIB_PATH = os.path.join(_HERE, '_build', 'libepic.so')
-NVCC_FLAGS = ['-gencode', 'arch=compute_103a,code=sm_103a', '-lineinfo', '-O3', '-std=c++17',
-              '-shared', '-Xcompiler', '-fPIC']
+ARCH_FLAGS = ['-gencode', 'arch=compute_103a,code=sm_103a']
+COMPILE_FLAGS = ARCH_FLAGS + ['-lineinfo', '-O3', '-std=c++17', '-Xcompiler', '-fPIC']
+NVCC_FLAGS = COMPILE_FLAGS + ['-shared']  # one-command form: nvcc NVCC_FLAGS sources -o lib
 
 OK, ERR_INVALID_ARG, ERR_GRAMMAR, ERR_LEXER, ERR_OOM, ERR_CUDA, ERR_CAPACITY, ERR_TIMEOUT = range(8)
 
@@ -32,17 +37,35 @@ class EpicError(RuntimeError):
         self.status = status
 
 
-def build(force: bool = False, verbose: bool = False) -> str:
-    """Compile the CUDA library for sm_103a (nvcc cross-compiles without a GPU)."""
+def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
+    """Compile the CUDA library for sm_103a (nvcc cross-compiles without a
+    GPU): every translation unit in parallel, then one link."""
     os.makedirs(os.path.dirname(LIB_PATH), exist_ok=True)
     newest = max(os.path.getmtime(p) for p in _DEPS)
     if force or not os.path.exists(LIB_PATH) or os.path.getmtime(LIB_PATH) < newest:
-        tmp = LIB_PATH + '.tmp%d' % os.getpid()
-        cmd = ['nvcc'] + NVCC_FLAGS + _SRC + ['-o', tmp]
-        if verbose:
-            print(' '.join(cmd))
-        subprocess.check_call(cmd)
-        os.replace(tmp, LIB_PATH)
+        tag = '%d' % os.getpid()
+        objs, procs = [], []
+        for src in _SRC:
+            obj = os.path.join(os.path.dirname(LIB_PATH), os.path.basename(src) + '.%s.o' % tag)
+            cmd = ['nvcc'] + COMPILE_FLAGS + list(extra_flags) + ['-c', src, '-o', obj]
+            if verbose:
+                print(' '.join(cmd))
+            procs.append((subprocess.Popen(cmd), cmd))
+            objs.append(obj)
+        failed = [cmd for p, cmd in procs if p.wait() != 0]
+        try:
+            if failed:
+                raise subprocess.CalledProcessError(1, failed[0])
+            tmp = LIB_PATH + '.tmp' + tag
+            cmd = ['nvcc'] + ARCH_FLAGS + ['-shared'] + objs + ['-o', tmp]
+            if verbose:
+                print(' '.join(cmd))
+            subprocess.check_call(cmd)
+            os.replace(tmp, LIB_PATH)
+        finally:
+            for o in objs:
+                if os.path.exists(o):
+                    os.remove(o)
     return LIB_PATH
 
 
