@@ -414,12 +414,19 @@ def test_monotonicity_and_witness(name):
 
 
 # ------------------------------------------------------------------ cover
-@pytest.mark.parametrize('gfun', [expr, tiny_paren, tiny_eps, G.json_grammar, G.smiles_grammar])
-def test_language_is_inside_the_cover(gfun):
-    g = gfun()
+COVER_GRAMMARS = {'expr': expr, 'tiny_paren': tiny_paren, 'tiny_eps': tiny_eps, 'json': G.json_grammar,
+                  'smiles': G.smiles_grammar, 'clike-512': lambda: G.grammar_for('clike-512'),
+                  'random-stress-1024': lambda: G.grammar_for('random-stress-1024')}
+
+
+@pytest.mark.parametrize('gname', list(COVER_GRAMMARS))
+def test_language_is_inside_the_cover(gname):
+    """L(G) inside L(F_G) (the cover over-approximates, App. D) on 10,000
+    sampled sentences per grammar."""
+    g = COVER_GRAMMARS[gname]()
     O = oracle.Oracle(g)
     rng = np.random.default_rng(1)
-    for _ in range(300):
+    for _ in range(10000):
         terms = sample_derivation(g, rng, int(rng.integers(1, 25)))
         assert O.accepts_terms(terms)
         assert O.cover_accepts_terms(terms)
