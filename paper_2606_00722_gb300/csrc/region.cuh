@@ -1,7 +1,11 @@
-// Validity checks by region, for grammars whose charts are large.
+// Validity checks by region, for grammars whose charts are large and for
+// batches with many checks per sequence.  The three steps live in
+// region_forward.cu, region_good.cu and region_check.cuh (instantiated by
+// region_check_sm.cu and region_check_global.cu).
 //
 // Every check x (+) (i, t) differs from x only around position i.  So:
-//  1. k_forward: one forward chart F of x per sequence (one warp each),
+//  1. k_forward: one forward chart F of x per sequence (one warp each; or
+//     k_forward_block, one CTA each),
 //     recording its graph (edges, gap flags), where each position's segment
 //     sits in it, and each entry's completed nonterminals.  If x itself is
 //     not completable, no single update is (the update's completion language
