@@ -90,3 +90,21 @@ def test_lex_table_runs_match_oracle(cuda, name):
             if r is not None:
                 ref.add(tuple(r[0]))
         assert mine == ref, (text, mine ^ ref)
+
+
+@pytest.mark.parametrize('shape', [(1, 16), (4, 4), (2, 8)])
+def test_pick_golden(cuda, shape):
+    """k_pick (Alg. 1's candidate set C) on the hand-derived golden cases,
+    bit for bit including the sign of a picked -0.0."""
+    import torch
+    import paper_2606_00722_gb300 as epic
+    from test_oracle_pins import load_pick_cases
+    valid, conf, cand, etok, econf = load_pick_cases()
+    B, k = shape
+    tok = torch.empty((B, k), dtype=torch.int32, device=cuda)
+    cf = torch.empty((B, k), dtype=torch.float32, device=cuda)
+    epic.pick_candidates(_dev(cand.reshape(B, k, 4), cuda), _dev(conf.reshape(B, k, 4), cuda),
+                         _dev(valid.reshape(B, k, 4), cuda), tok, cf)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(tok.cpu().numpy().reshape(-1), etok)
+    np.testing.assert_array_equal(cf.cpu().numpy().reshape(-1).view(np.uint32), econf.view(np.uint32))

@@ -530,3 +530,123 @@ def test_commit_writes_selected_tokens():
     sel = np.array([[1, 0], [1, 1]], np.uint8)
     y = oracle.Oracle.commit(x, pos, tok, sel)
     assert y[0, 0] == 7 and y[0, 3] == -1 and y[1, 1] == 9 and y[1, 2] == 10
+
+
+# ------------------------------------------------------------------ candidate set C
+def load_pick_cases():
+    """tests/golden/pick_cases.txt as (valid [R][4], conf [R][4], cand [R][4],
+    expected token [R], expected confidence [R]); token of line r, index c is
+    100 r + c."""
+    rows = []
+    with open(os.path.join(HERE, 'golden', 'pick_cases.txt')) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith('#'):
+                continue
+            v, c, t, e = (s.strip() for s in line.split('|'))
+            rows.append(([int(a) for a in v.split()], [float(a) for a in c.split()], int(t), float(e)))
+    R = len(rows)
+    valid = np.array([r[0] for r in rows], np.uint8)
+    conf = np.array([r[1] for r in rows], np.float32)
+    cand = (100 * np.arange(R)[:, None] + np.arange(4)[None, :]).astype(np.int32)
+    return valid, conf, cand, np.array([r[2] for r in rows], np.int32), np.array([r[3] for r in rows], np.float32)
+
+
+@pytest.mark.parametrize('shape', [(1, 16), (4, 4), (2, 8)])
+def test_pick_candidates_golden(shape):
+    """Alg. 1's candidate set C on hand-derived cases: highest confidence among
+    valid-bit-1 candidates, ties to the lowest index, overflow (2) never
+    picked, none -> (-1, 0.0), -0.0 ties with 0.0 (the sign of the picked
+    value is kept).  The rows are laid out as several batch shapes so that a
+    transposed (sequence, position) index fails."""
+    valid, conf, cand, etok, econf = load_pick_cases()
+    B, k = shape
+    assert B * k == len(etok)
+    tok, cf = oracle.pick_candidates(valid.reshape(B, k, 4), cand.reshape(B, k, 4), conf.reshape(B, k, 4))
+    np.testing.assert_array_equal(tok.reshape(-1), etok)
+    np.testing.assert_array_equal(cf.reshape(-1).view(np.uint32), econf.view(np.uint32))
+
+
+# ------------------------------------------------------------------ cover on partial outputs
+def all_partials(vocab_n, n):
+    for x in itertools.product(range(-1, vocab_n), repeat=n):
+        yield np.array(x, np.int32)
+
+
+def test_cover_valid_equals_valid_when_the_cover_is_exact():
+    """tiny_nonrec's cover is exact (no recursion, no nonterminal used twice:
+    L(F_G) = L(G), App. D.3), so on every partial output -- gaps included --
+    the cover test 1[L(F_G) cap C_x != empty] and the exact test
+    1[L(G) cap C_x != empty] of Sec. 3 must agree: both over- and
+    under-acceptance of the cover's gap closure fail here."""
+    g = tiny_nonrec()
+    vocab = [b'a', b'b', b'c', b'd', b'e', b'ad', b'ab', b'ce']
+    O = oracle.Oracle(g, vocab)
+    n_valid = n_cover = 0
+    for n in range(0, 5):
+        for x in all_partials(len(vocab), n):
+            v = O.valid(x)
+            assert O.cover_valid(x) == v, x
+            n_valid += v
+            n_cover += 1
+    rng = np.random.default_rng(9)
+    for _ in range(3000):
+        x = random_partial(rng, len(vocab), int(rng.integers(5, 9)), 0.4)
+        assert O.cover_valid(x) == O.valid(x), x
+    assert 0 < n_valid < n_cover
+
+
+def _paren_runs(vocab, x):
+    """Terminal view of a tiny_paren partial output whose tokens are made of
+    the one-character terminals and skipped spaces: the fixed runs between
+    gaps (as terminal-name strings) and whether each boundary is a gap."""
+    segs, cur, gaps = [], '', []
+    for t in x:
+        if t < 0:
+            if not gaps or not gaps[-1][1] or cur:
+                segs.append(cur)
+                gaps.append((len(segs) - 1, True))
+                cur = ''
+        else:
+            cur += vocab[t].decode().replace(' ', '')
+    segs.append(cur)
+    return segs, sum(1 for _ in gaps)
+
+
+def test_cover_valid_brute_force_over_gap_fillings():
+    """tiny_paren (recursive; its cover over-accepts): the cover test of a
+    partial output holds iff some filling of its gaps with terminal strings is
+    accepted by the cover as a plain string.  The fillings are enumerated up
+    to length 4 (one gap) or 3 (two gaps), over the terminals that occur in
+    productions; the cover has few enough states that any state reachable
+    across a gap is reachable within that length."""
+    g = tiny_paren()
+    vocab = [b'(', b')', b'a', b'b', b' ', b'((', b'a)', b' (']
+    O = oracle.Oracle(g, vocab)
+    idx = {t.name: i for i, t in enumerate(g.terminals)}
+    fills = {L: [''.join(s) for m in range(L + 1) for s in itertools.product('()a', repeat=m)] for L in (3, 4)}
+    cache = {}
+
+    def cover_str(s):
+        if s not in cache:
+            cache[s] = O.cover_accepts_terms([idx[c] for c in s])
+        return cache[s]
+
+    checked = agree_true = 0
+    for n in range(1, 5):
+        for x in all_partials(len(vocab), n):
+            segs, ngaps = _paren_runs(vocab, x)
+            if ngaps > 2:
+                continue
+            L = 4 if ngaps <= 1 else 3
+            if ngaps == 0:
+                expect = cover_str(segs[0])
+            elif ngaps == 1:
+                expect = any(cover_str(segs[0] + f + segs[1]) for f in fills[L])
+            else:
+                expect = any(cover_str(segs[0] + f1 + segs[1] + f2 + segs[2])
+                             for f1 in fills[L] for f2 in fills[L])
+            assert O.cover_valid(x) == expect, (x, segs)
+            checked += 1
+            agree_true += expect
+    assert checked > 3000 and 0 < agree_true < checked
