@@ -156,17 +156,22 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
  * -- a serving process that has handed all device memory to its own pool
  * (model weights, KV cache) before decoding starts, or a per-step decode
  * loop that must not take cudaMalloc's implicit device synchronization and
- * unbounded latency.  Same arguments, outputs and errors as
- * epic_validate_batch; results are identical.
+ * unbounded latency.  Same arguments and outputs as epic_validate_batch;
+ * every check that neither call reports as overflow (2) gets the same bit.
+ * It always walks each check's whole graph (never by region), so it may
+ * additionally report 2 where epic_validate_batch answers, and it has two
+ * extra capacity errors, both returned before anything is enqueued:
+ *   - EPIC_ERR_CAPACITY when the grammar's item sets exceed 32 words and
+ *     n > 128 (whole-graph walks of long rows of such grammars take
+ *     seconds per check; use epic_validate_batch for them);
+ *   - EPIC_ERR_CAPACITY when one walk's workspace, (8 n + 256) columns and
+ *     256 n chart entries, does not fit in the array.
+ * A check whose chart needs more than 256 n entries reports 2 (overflow).
+ * Fewer walks run at once than in epic_validate_batch, so it is slower on
+ * large batches.
  *
  * Scratch: a file-scope device array of 128 MiB inside the library, which
- * every GPU that loads the library holds until the process exits.  Each
- * walk needs (8 n + 256) columns and 256 n chart entries of workspace; if
- * one walk's workspace does not fit in the array (long sequences with a
- * wide grammar) the call returns EPIC_ERR_CAPACITY before enqueueing
- * anything, and a check whose chart needs more than 256 n entries reports
- * 2 (overflow) in d_valid.  Fewer walks run at once than in
- * epic_validate_batch, so it is slower on large batches.
+ * every GPU that loads the library holds until the process exits.
  * The first call on a device looks up the array's device address (once per
  * device, with that device current); make that first call before any
  * stream capture.  Every call on a device shares the one array and keeps

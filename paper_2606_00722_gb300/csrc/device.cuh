@@ -32,6 +32,11 @@ struct DevGrammar {
   const int32_t* dfa_next;        // [Q][256]
   const uint8_t* dfa_ext;         // [Q] 1 if some byte continues the lexeme
   const uint8_t* skip;            // [T]
+  // advance closure by doubling: adv_pow[m][s][w] (m = 0: nullable_next,
+  // m = 1: next_any) holds the items i with i .. i + 2^s - 1 all in the mask;
+  // adv_steps doublings cover the longest production
+  const uint32_t* adv_pow;        // [2][adv_steps][W]
+  int adv_steps;
   // regular cover (flattened RTN), see cover.cuh
   int FS, FW;                     // cover states and words
   const uint32_t* cov_eps_close;  // [FS][FW] epsilon closure of each state

@@ -11,6 +11,7 @@
 #include <vector>
 
 #include "../../include/epic.h"
+#include "../../include/epic_measure.h"
 #include "grammar.h"
 #include "launch.h"
 
@@ -128,7 +129,20 @@ struct epic_lexer_table {
   long long wemax = 0;
   int wwarps = 0;
   cudaStream_t last = nullptr;
+  // CUDA events around the kernels of the last epic_validate_batch call
+  // (epic_last_kernel_times): kev[i] .. kev[i + 1] is kernel i
+  cudaEvent_t kev[4] = {nullptr, nullptr, nullptr, nullptr};
+  int nk = 0;
+  const char* kname[3] = {nullptr, nullptr, nullptr};
 };
+
+namespace {
+// record event i of the table's kernel timing on st (created on first use)
+void mark(epic_lexer_table* t, int i, cudaStream_t st) {
+  if (!t->kev[i] && cudaEventCreate(&t->kev[i]) != cudaSuccess) t->kev[i] = nullptr;
+  if (t->kev[i]) cudaEventRecord(t->kev[i], st);
+}
+}  // namespace
 
 namespace {
 
@@ -273,7 +287,7 @@ epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const in
   const DevGrammar& dg = g->dg;
   long long total = (long long)B * k * K;
   SeqPack sp;
-  sp.nmax = std::min(1900, 8 * n + 256);
+  sp.nmax = std::min(kMaxCols, 8 * n + 256);
   sp.n = n;
   sp.W = dg.W;
   sp.VW = dg.VW;
@@ -330,10 +344,17 @@ epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const in
     int wpc = kWarpsPerCta;
     size_t per = smem_per_warp(sp.nmax, rmax, dg.W, dg.VW);
     if (sm) wpc = (int)std::min<size_t>(kWarpsPerCta, smem_cap / per);
-    bool block_walk = false;
-    if (const char* e = getenv("EPIC_FORWARD_BLOCK")) block_walk = atoi(e) != 0;
-    if (block_walk) {
-      launch_forward_block(B, st, dg, t->d_table, t->vocab, d_x, B, n, sp, t->d_stats);
+    // wide item sets: one CTA per sequence (Gauss-Seidel columns); narrow
+    // ones: one warp per sequence.  EPIC_FORWARD_CTA=0/1 overrides.
+    bool cta_walk = dg.W > 32;
+    if (const char* e = getenv("EPIC_FORWARD_CTA")) cta_walk = atoi(e) != 0;
+    t->nk = 3;
+    t->kname[0] = cta_walk ? "k_forward_gs" : "k_forward";
+    t->kname[1] = "k_good";
+    t->kname[2] = "k_check";
+    mark(t, 0, st);
+    if (cta_walk) {
+      launch_forward_gs(std::min(B, 4 * sm_count()), st, dg, t->d_table, t->vocab, d_x, B, n, sp, t->d_stats);
     } else if (sm && wpc >= 1) {
       size_t dyn = per * wpc;
       launch_forward(true, (B + wpc - 1) / wpc, 32 * wpc, dyn, st, dg, t->d_table, t->vocab, d_x, B, n, sp, rmax,
@@ -344,7 +365,9 @@ epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const in
     }
   }
   // 2. good masks
+  mark(t, 1, st);
   launch_good(B, st, dg, B, sp);
+  mark(t, 2, st);
   t->n_region += total;
   t->n_vkernels += 3;
   // 3. checks
@@ -363,6 +386,7 @@ epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const in
     launch_check_global(blocks, 32 * per_cta, 0, st, dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K, total,
                         d_valid, sp, wp, t->d_regs, 0, t->d_counter, t->d_stats);
   }
+  mark(t, 3, st);
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
 }
 
@@ -504,6 +528,30 @@ epic_status epic_grammar_create(const epic_grammar_desc* desc, epic_grammar** ou
       if (g->dfa.next[(size_t)q * 256 + c] >= 0) ext[q] = 1;
   up(ext, &d.dfa_ext);
   up(G.skip, &d.skip);
+  {
+    // runs of advanceable items for the doubling closure (see device.cuh)
+    int maxlen = 0;
+    for (size_t p = 0; p + 1 < G.rhs_off.size(); ++p) maxlen = std::max(maxlen, G.rhs_off[p + 1] - G.rhs_off[p]);
+    int steps = 1;
+    while ((1 << steps) <= maxlen) ++steps;
+    d.adv_steps = steps;
+    std::vector<uint32_t> pw((size_t)2 * steps * G.W, 0);
+    auto bit = [&](const std::vector<uint32_t>& m, long long i) -> bool {
+      return i >= 0 && i < (long long)G.W * 32 && ((m[(size_t)(i >> 5)] >> (i & 31)) & 1u);
+    };
+    for (int mode = 0; mode < 2; ++mode) {
+      std::vector<uint32_t> cur = mode ? next_any : G.nullable_next;
+      for (int st2 = 0; st2 < steps; ++st2) {
+        std::copy(cur.begin(), cur.end(), pw.begin() + ((size_t)mode * steps + st2) * G.W);
+        const long long k = 1ll << st2;  // next: i and i + k both start runs of length k
+        std::vector<uint32_t> nx(G.W, 0);
+        for (long long i = 0; i < (long long)G.W * 32; ++i)
+          if (bit(cur, i) && bit(cur, i + k)) nx[(size_t)(i >> 5)] |= 1u << (i & 31);
+        cur.swap(nx);
+      }
+    }
+    up(pw, &d.adv_pow);
+  }
   d.FS = g->cov.FS;
   d.FW = g->cov.FW;
   d.cov_start = g->cov.start;
@@ -593,6 +641,8 @@ void epic_lexer_table_destroy(epic_lexer_table* t) {
   cudaFree(t->d_regs);
   cudaFree(t->d_stats);
   cudaFree(t->d_counter);
+  for (cudaEvent_t e : t->kev)
+    if (e) cudaEventDestroy(e);
   delete t;
 }
 
@@ -645,6 +695,9 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
   int per_sm = (int)((t->wwarps + sm_count() - 1) / sm_count());
   if (wpc > per_sm) wpc = std::max(2, per_sm);
   t->n_vkernels += 1;
+  t->nk = 1;
+  t->kname[0] = "k_validate_warp";
+  mark(t, 0, st);
   if (wpc >= 2) {
     size_t dyn = per * wpc + (gsm ? gt : 0);
     int blocks = (t->wwarps + wpc - 1) / wpc;
@@ -655,7 +708,22 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
     launch_validate_warp(false, t->wwarps / kWarpsPerCta, 32 * kWarpsPerCta, 0, st, g->dg, t->d_table, t->vocab, d_x,
                          n, d_pos, k, d_cand, K, total, d_valid, wp, 0, 0, t->d_counter, t->d_stats);
   }
+  mark(t, 1, st);
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
+}
+
+int epic_last_kernel_times(const epic_lexer_table* t, float* ms, const char** names, int cap) {
+  if (!t || (!ms && cap > 0) || cap < 0) return -1;
+  const int n = std::min(t->nk, cap);
+  for (int i = 0; i <= t->nk; ++i)
+    if (!t->kev[i]) return -1;
+  if (t->nk == 0) return 0;
+  if (cudaEventSynchronize(t->kev[t->nk]) != cudaSuccess) return -1;
+  for (int i = 0; i < n; ++i) {
+    if (cudaEventElapsedTime(&ms[i], t->kev[i], t->kev[i + 1]) != cudaSuccess) return -1;
+    if (names) names[i] = t->kname[i];
+  }
+  return n;
 }
 
 }  // extern "C"
@@ -665,6 +733,7 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
 // which loads this library holds until the process exits.  Its first 256
 // bytes hold the work counter; the rest is carved into per-warp workspaces.
 constexpr size_t kNoAllocBytes = (size_t)128 << 20;
+constexpr int kNoAllocWideMaxN = 128;  // row length limit when item sets exceed 32 words
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
 
 namespace {
@@ -674,9 +743,10 @@ void* g_noalloc_ptr[256] = {nullptr};  // device address of the array, per devic
 
 extern "C" {
 
-epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_table* t, const int32_t* d_x,
+epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_table* tc, const int32_t* d_x,
                                         int32_t B, int32_t n, const int32_t* d_pos, int32_t k,
                                         const int32_t* d_cand, int32_t K, uint8_t* d_valid, void* cuda_stream) {
+  epic_lexer_table* t = const_cast<epic_lexer_table*>(tc);
   if (!g || !t || t->g != g || B < 0 || n < 0 || k < 0 || K < 0) return EPIC_ERR_INVALID_ARG;
   long long total = (long long)B * k * K;
   if (total == 0) return EPIC_OK;
@@ -697,6 +767,11 @@ epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_
     base = (char*)g_noalloc_ptr[dev];
   }
   const int W = g->dg.W, VW = g->dg.VW;
+  // Wide item sets walk the whole graph per check with rows in the global
+  // stage, which takes seconds per check on long rows of large grammars; the
+  // fixed array holds too few walks for that to finish in reasonable time,
+  // so such calls are limited to short rows.
+  if (W > 32 && n > kNoAllocWideMaxN) return EPIC_ERR_CAPACITY;
   WPack wp;
   wp.base = base + 256;
   wp.nmax = std::min(kWCols, 8 * n + 256);
@@ -711,6 +786,9 @@ epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_
   size_t sper = smem_per_warp(wp.nmax, rmax, W, VW);
   int wpc = (W > 32) ? 0 : (int)std::min<size_t>(kWarpsPerCta, smem_cap / sper);
   unsigned long long* counter = (unsigned long long*)base;
+  // the kernel reads the table's lex entries and adds into its counters:
+  // epic_get_stats and epic_lexer_table_destroy synchronize this stream
+  t->last = st;
   if (cudaMemsetAsync(counter, 0, sizeof(unsigned long long), st) != cudaSuccess) return EPIC_ERR_CUDA;
   t->n_vkernels += 1;
   if (wpc >= 2) {

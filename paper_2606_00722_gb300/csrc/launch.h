@@ -21,8 +21,8 @@ void launch_validate_warp(bool sm, dim3 grid, dim3 block, size_t dyn, cudaStream
 void launch_forward(bool sm, dim3 grid, dim3 block, size_t dyn, cudaStream_t st, const DevGrammar& g,
                     const LexEntry* table, int vocab, const int32_t* x, int B, int n, const SeqPack& sp, int rmax,
                     unsigned long long* stats);
-void launch_forward_block(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab,
-                          const int32_t* x, int B, int n, const SeqPack& sp, unsigned long long* stats);
+void launch_forward_gs(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab,
+                       const int32_t* x, int B, int n, const SeqPack& sp, unsigned long long* stats);
 void launch_good(dim3 grid, cudaStream_t st, const DevGrammar& g, int B, const SeqPack& sp);
 void launch_check_sm(dim3 grid, dim3 block, size_t dyn, cudaStream_t st, const DevGrammar& g, const LexEntry* table,
                      int vocab, const int32_t* x, int n, const int32_t* pos, int k, const int32_t* cand, int K,

@@ -82,6 +82,7 @@ struct WPack {
     ws.g_end = (int32_t*)take(kWMaxQ * 4);
     ws.g_len = (int32_t*)take(kWMaxQ * 4);
     ws.g_last = (int32_t*)take(kWMaxQ * 4);
+    ws.key_q = (int32_t*)take(kWMaxQ * 4);
     ws.g_tail = (uint32_t*)take(kWMaxQ * 16);
     ws.g_lbl = (uint32_t*)take(kWMaxQ * 32);
     ws.ssum = (uint32_t*)take((size_t)nmax * 8);
@@ -94,7 +95,7 @@ struct WPack {
 
 inline size_t wbytes_per_warp(int nmax, long long emax, int W, int VW) {
   auto r = [](size_t b) { return (b + 255) & ~(size_t)255; };
-  return r((size_t)nmax * W * 4) + r((size_t)nmax * VW * 4) + r((size_t)(nmax + 1) * 4) + 6 * r(kWMaxQ * 4) +
+  return r((size_t)nmax * W * 4) + r((size_t)nmax * VW * 4) + r((size_t)(nmax + 1) * 4) + 7 * r(kWMaxQ * 4) +
          r(kWMaxQ * 16) + r(kWMaxQ * 32) + r((size_t)nmax * 8) + r((size_t)emax * 4) + r((size_t)emax * 8) +
          r((size_t)emax * W * 4);
 }

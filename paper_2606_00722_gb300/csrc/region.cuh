@@ -25,6 +25,7 @@
 //     good item is found (or the accepting item, when the region holds the
 //     start or the end).
 #pragma once
+#include "gscols.cuh"
 #include "packs.cuh"
 #include "seqpack.cuh"
 

@@ -64,19 +64,22 @@ __global__ void __launch_bounds__(32 * kWarpsPerCta) k_forward(DevGrammar g, con
   }
 }
 
-// The same forward charts with a whole CTA per sequence: the block walk
-// spreads each closure round's dirty origins and completion pairs over the
-// warps (for long sequences of wide grammars, where one warp's walk is a long
-// serial chain).  Selected with EPIC_FORWARD_BLOCK=1.
-__global__ void __launch_bounds__(kThreads) k_forward_block(DevGrammar g, const LexEntry* __restrict__ table,
-                                                            int vocab, const int32_t* __restrict__ x, int B, int n,
-                                                            SeqPack sp, unsigned long long* stats) {
+// The same forward charts with a whole CTA per sequence (wide grammars,
+// long rows): the Gauss-Seidel column closure of gscols.cuh, the CTA
+// scattering each origin's completions.  The grammar's per-item tables sit in
+// dynamic shared memory.
+__global__ void __launch_bounds__(32 * kGsMaxWarps, 1) k_forward_gs(DevGrammar g, const LexEntry* __restrict__ table,
+                                                                    int vocab, const int32_t* __restrict__ x, int B,
+                                                                    int n, SeqPack sp, unsigned long long* stats) {
   __shared__ WalkShared sh;
+  __shared__ GsShared gss;
+  extern __shared__ __align__(16) unsigned char dyn[];
+  GsTables tb;
+  gs_stage_tables(g, dyn, tb);
   for (long long b = blockIdx.x; b < B; b += gridDim.x) {
     SeqArena a = sp.carve(b);
-    // the walk expects a zeroed stage and completion record
+    // the walk expects a zeroed stage
     for (size_t w = threadIdx.x; w < (size_t)sp.nmax * g.W; w += blockDim.x) a.ws.stage[w] = 0;
-    for (size_t w = threadIdx.x; w < (size_t)sp.nmax * g.VW; w += blockDim.x) a.ws.bdone[w] = 0;
     for (int p = threadIdx.x; p < n; p += blockDim.x) {
       a.rec.gap_col[p] = -1;
       a.rec.pre_col[p] = -1;
@@ -85,7 +88,7 @@ __global__ void __launch_bounds__(kThreads) k_forward_block(DevGrammar g, const 
     __syncthreads();
     Workspace ws;
     ws.stage = a.ws.stage;
-    ws.bdone = a.ws.bdone;
+    ws.bdone = nullptr;
     ws.col_off = a.ws.col_off;
     ws.org = a.ws.org;
     ws.bits = a.ws.bits;
@@ -100,16 +103,16 @@ __global__ void __launch_bounds__(kThreads) k_forward_block(DevGrammar g, const 
     sc.f_q = a.ws.f_q;
     sc.f_c = a.ws.f_c;
     sc.key_q = a.key_q;
-    sc.expn = a.bexpn;
-    sc.bnew = a.bnew;
+    sc.expn = nullptr;
+    sc.bnew = nullptr;
     const BlockRec br{a.rec.col_gap, a.rec.e_dst,   a.rec.e_src,   a.rec.e_lbl,    a.rec.cnt,
                       a.ws.esum,     a.rec.gap_col, a.rec.pre_col, a.rec.post_col, a.rec.edge_cap};
     WsDims d;
     d.nmax = sp.nmax;
     d.emax = sp.emax;
-    EarleyColsT<true> cols(g, table, ws, sc, d, sh);
+    EarleyColsGS<true> cols(g, tb, table, ws, sc, d, sh, gss);
     cols.rec = &br;
-    Walk<EarleyColsT<true>> walk(cols, g, table, sc, sh, vocab);
+    Walk<EarleyColsGS<true>> walk(cols, g, table, sc, sh, vocab);
     walk.rec = &br;
     Subst none{nullptr, nullptr, 0};
     const int r = walk.run(x + b * n, n, none);
@@ -129,7 +132,6 @@ __global__ void __launch_bounds__(kThreads) k_forward_block(DevGrammar g, const 
   }
 }
 
-
 void launch_forward(bool sm, dim3 grid, dim3 block, size_t dyn, cudaStream_t st, const DevGrammar& g,
                     const LexEntry* table, int vocab, const int32_t* x, int B, int n, const SeqPack& sp, int rmax,
                     unsigned long long* stats) {
@@ -141,9 +143,11 @@ void launch_forward(bool sm, dim3 grid, dim3 block, size_t dyn, cudaStream_t st,
   }
 }
 
-void launch_forward_block(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab,
-                          const int32_t* x, int B, int n, const SeqPack& sp, unsigned long long* stats) {
-  k_forward_block<<<grid, kThreads, 0, st>>>(g, table, vocab, x, B, n, sp, stats);
+void launch_forward_gs(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab,
+                       const int32_t* x, int B, int n, const SeqPack& sp, unsigned long long* stats) {
+  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps);
+  cudaFuncSetAttribute(k_forward_gs, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+  k_forward_gs<<<grid, 32 * kGsMaxWarps, dyn, st>>>(g, table, vocab, x, B, n, sp, stats);
 }
 
 // measurement builds: this translation unit's phase counters of the walk

@@ -15,7 +15,31 @@ __device__ __forceinline__ uint32_t shr1_word(const uint32_t* src, int w, int W)
   return v;
 }
 
-constexpr int kGoodWarps = 32;  // one CTA per sequence
+constexpr int kGoodWarps = 16;  // one CTA per sequence
+
+// Warp, row in registers: r |= bits & M & shr1(r) until stable -- an item is
+// good when it may advance within its own row and the advanced item is good.
+template <int KW>
+__device__ __forceinline__ void good_in_row(uint32_t (&r)[KW], const uint32_t (&bits)[KW], const uint32_t (&M)[KW],
+                                            int W) {
+  const int lane = threadIdx.x & 31;
+  for (int it = 0; it < 64; ++it) {
+    bool ch = false;
+#pragma unroll
+    for (int i = 0; i < KW; ++i) {
+      if (32 * i >= W) break;
+      // bit b of word w takes bit b+1 (bit 0 of word w+1 for b = 31)
+      uint32_t nxt = __shfl_down_sync(0xffffffffu, r[i], 1);
+      const uint32_t wrap = (i + 1 < KW) ? __shfl_sync(0xffffffffu, r[i + 1], 0) : 0u;
+      if (lane == 31) nxt = wrap;
+      const uint32_t s = (r[i] >> 1) | (nxt << 31);
+      const uint32_t add = bits[i] & M[i] & s & ~r[i];
+      ch |= add != 0;
+      r[i] |= add;
+    }
+    if (!__any_sync(0xffffffffu, ch)) break;
+  }
+}
 
 // Good items of a sequence's forward chart, columns from last to first.
 // Item i of entry (j, o) is good when it is present and
@@ -27,23 +51,32 @@ constexpr int kGoodWarps = 32;  // one CTA per sequence
 //  - j is a gap and the item advanced over any symbol is good;
 //  - it is complete with left side B, and some item of column o, origin o2,
 //    waiting on B has its advanced item good at (j, o2).
-// The first three read later columns only (final); the last two read this
-// column: its entries iterate to the least fixpoint together.
+// The first three read later columns only (final); the in-row ones (gap,
+// nullable) close each row on its own.  The last one reads entries (j, o2)
+// of this column with o2 <= o, so the entries holding complete items are
+// closed in ascending origin order, once each: the whole CTA gathers which
+// completed nonterminals of (j, o) some waiting item of column o turns good,
+// then one warp closes (j, o) with its own self-loop (the entry of column o
+// with origin o maps back to (j, o)).
 __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B, SeqPack sp) {
-  const long long b = blockIdx.x;
-  if (b >= B) return;
+  extern __shared__ __align__(16) unsigned char dyn[];
+  GsTables tb;
+  gs_stage_tables(g, dyn, tb);
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nthr = blockDim.x;
   const int W = g.W, VW = g.VW;
+  constexpr int KW = kWMaxW / 32;  // item words per lane
+  __shared__ int s_self;
+  __shared__ uint32_t s_cn[kWMaxVW], s_bset[kWMaxVW];
+  __shared__ uint32_t s_expn[kWMaxW];
+  __shared__ int s_flag;
+  for (long long b = blockIdx.x; b < B; b += gridDim.x) {
   SeqArena a = sp.carve(b);
   int32_t* meta = a.rec.meta;
-  if (meta[M_STATUS] != 1) return;
+  if (meta[M_STATUS] != 1) continue;
   const int N = meta[M_NCOLS], NE = meta[M_NEDGES];
   const int32_t* col = a.ws.col_off;
   const int32_t* org = a.ws.org;
   const int start = meta[M_START], accept = meta[M_ACCEPT];
-  __shared__ int s_flag, s_self;
-  __shared__ uint32_t s_nt[kGoodWarps][kWMaxVW];
-  constexpr int KW = kWMaxW / 32;  // item words per lane
   int32_t* cur_o = a.cursor;          // [N + 1]
   int32_t* cur_s = a.cursor + N + 1;  // [N + 1]
   // edges by source and entries by origin (CSR), entry index by (column, origin)
@@ -88,7 +121,6 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
 
   uint32_t* G = a.good;
   uint32_t* sfold = (uint32_t*)a.cursor;  // per successor of the column (the cursors are free now)
-  const int nwl = (W + 31) >> 5;          // item words per lane in use
   for (int j = N - 1; j >= 0; --j) {
     const int s0 = a.succ_off[j], s1 = a.succ_off[j + 1];
     const bool gap = a.rec.col_gap[j] != 0;
@@ -104,23 +136,36 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
     for (int si = s0 + warp; si < s1; si += kGoodWarps) {
       const int j2 = a.succ_idx[si];
       const uint32_t* cn = a.rec.cnt + (size_t)a.eidx[tri_index(j2, j)] * VW;
-      expn_of_set(g, cn, a.expn + (size_t)(si - s0) * W);
-      if (lane == 0) {  // folded set (bit C mod 32): a filter against an entry's waited nonterminals
-        uint32_t f = 0;
-        for (int v = 0; v < VW; ++v) f |= cn[v];
-        sfold[si - s0] = f;
-      }
+      uint32_t f = 0;
+      for (int v = 0; v < VW; ++v) f |= cn[v];
+      if (f) expn_of_set(g, cn, a.expn + (size_t)(si - s0) * W);
+      if (lane == 0) sfold[si - s0] = f;  // folded (bit C mod 32): 0 = nothing completes
     }
     __syncthreads();
-    // from the later columns: scans along the out-edges, nested constituents
-    // (the lanes look up 32 successor columns at a time)
+    // in-row rules of this column: the gap self-loop and nullable completions
+    uint32_t inrow[KW];
+#pragma unroll
+    for (int i = 0; i < KW; ++i) {
+      const int w = lane + 32 * i;
+      uint32_t m = 0;
+      if (w < W) {
+        if (gap) m |= tb.next_any[w];
+        if (self_si >= 0 && sfold[self_si]) m |= a.expn[(size_t)self_si * W + w];
+      }
+      inrow[i] = m;
+    }
+    // A. the rules that read later columns, then the in-row closure (one warp
+    //    per entry)
     for (long long k = k0 + warp; k < k1; k += kGoodWarps) {
       const int o = org[k];
-      const uint32_t* bits = a.ws.bits + (size_t)k * W;
-      uint32_t* Gk = G + (size_t)k * W;
-      uint32_t acc[KW];
+      const uint32_t* bp = a.ws.bits + (size_t)k * W;
+      uint32_t acc[KW], bits[KW];
 #pragma unroll
-      for (int i = 0; i < KW; ++i) acc[i] = 0;
+      for (int i = 0; i < KW; ++i) {
+        const int w = lane + 32 * i;
+        acc[i] = 0;
+        bits[i] = (w < W) ? bp[w] : 0u;
+      }
       if (j == accept && o == start && lane == ((g.accept_item >> 5) & 31))
         acc[g.accept_item >> 10] |= 1u << (g.accept_item & 31);
       for (int ei = a.out_off[j]; ei < a.out_off[j + 1]; ++ei) {
@@ -137,7 +182,6 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
         }
 #pragma unroll
         for (int i = 0; i < KW; ++i) {
-          if (i >= nwl) break;
           const int w = lane + 32 * i;
           if (w < W) {
             if (eps) {
@@ -175,108 +219,157 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
           const uint32_t* G3 = G + (size_t)kk * W;
 #pragma unroll
           for (int i = 0; i < KW; ++i) {
-            if (i >= nwl) break;
             const int w = lane + 32 * i;
-            if (w < W) acc[i] |= ex[w] & shr1_word(G3, w, W);
+            if (w < W) {
+              const uint32_t xw = ex[w];
+              if (xw) acc[i] |= xw & shr1_word(G3, w, W);
+            }
           }
         }
       }
+#pragma unroll
+      for (int i = 0; i < KW; ++i) acc[i] &= bits[i];
+      good_in_row<KW>(acc, bits, inrow, W);
       bool nz = false;
+      uint32_t* Gk = G + (size_t)k * W;
 #pragma unroll
       for (int i = 0; i < KW; ++i) {
         const int w = lane + 32 * i;
-        if (w < W) {
-          const uint32_t v = bits[w] & acc[i];
-          Gk[w] = v;
-          nz |= v != 0;
-        }
+        if (w < W) Gk[w] = acc[i];
+        nz |= acc[i] != 0;
       }
       nz = __any_sync(0xffffffffu, nz);
       if (lane == 0) a.gnz[k] = nz ? 1 : 0;
     }
     __syncthreads();
-    // completions within the column and the self rules, to the fixpoint
-    for (int pass = 0;; ++pass) {
-      if (pass > (1 << 20)) {  // cannot happen before the fixpoint; never silently wrong
-        if (tid == 0) meta[M_STATUS] = -1;
-        return;
+    // B. completions within the column, entries with complete items in
+    //    ascending origin order
+    for (long long k = k0; k < k1; ++k) {
+      const int o = org[k];
+      const uint32_t* cn = a.rec.cnt + (size_t)k * VW;
+      for (int v = tid; v < VW; v += nthr) {
+        s_cn[v] = cn[v];
+        s_bset[v] = 0;
       }
-      if (tid == 0) s_flag = 0;
+      if (tid == 0) {
+        uint32_t f = 0;
+        for (int v = 0; v < VW; ++v) f |= cn[v];
+        s_flag = f != 0;
+      }
       __syncthreads();
-      bool changed = false;
-      uint32_t* bset = s_nt[warp];
-      for (long long k = k0 + warp; k < k1; k += kGoodWarps) {
-        const int o = org[k];
-        const uint32_t* bits = a.ws.bits + (size_t)k * W;
+      if (!s_flag) continue;  // no complete item here
+      // items waiting on a nonterminal completed at (j, o)
+      for (int w = tid; w < W; w += nthr) {
+        uint32_t acc = 0, m = tb.any_nt[w];
+        while (m) {
+          const int bb = __ffs(m) - 1;
+          m &= m - 1;
+          const int Bn = tb.item_next[(w << 5) + bb] - g.T;
+          if ((s_cn[Bn >> 5] >> (Bn & 31)) & 1u) acc |= 1u << bb;
+        }
+        s_expn[w] = acc;
+      }
+      __syncthreads();
+      // which of them some entry (o, o2 < o) of column o turns good at (j, o2)
+      const int cb = col[o], ce = col[o + 1];
+      const bool self = ce > cb && org[ce - 1] == o;
+      const int nent = self ? ce - cb - 1 : ce - cb;
+      const long long total = (long long)nent * W;
+      for (long long t = tid; t < total; t += nthr) {
+        const int kp = cb + (int)(t / W), w = (int)(t % W);
+        const int kk = a.eidx[tri_index(j, org[kp])];
+        if (kk < 0 || !a.gnz[kk]) continue;
+        uint32_t m = a.ws.bits[(size_t)kp * W + w] & s_expn[w] & shr1_word(G + (size_t)kk * W, w, W);
+        while (m) {
+          const int bb = __ffs(m) - 1;
+          m &= m - 1;
+          const int Bn = tb.item_next[(w << 5) + bb] - g.T;
+          const uint32_t bit = 1u << (Bn & 31);
+          if (!(s_bset[Bn >> 5] & bit)) atomicOr(&s_bset[Bn >> 5], bit);
+        }
+      }
+      __syncthreads();
+      // one warp: complete items with a good left side, the in-row closure,
+      // and the self-loop through the entry of column o with origin o
+      if (warp == 0) {
+        const uint32_t* bp = a.ws.bits + (size_t)k * W;
+        const uint32_t* E = self ? a.ws.bits + (size_t)(ce - 1) * W : nullptr;
         uint32_t* Gk = G + (size_t)k * W;
-        // each round that changes the entry adds an item
-        for (int round = 0; round <= W * 32; ++round) {
-          for (int v = lane; v < VW; v += 32) bset[v] = 0;
-          __syncwarp();
-          for (long long kb = col[o]; kb < col[o + 1]; kb += 32) {  // 32 lookups at a time
-            const long long kp = kb + lane;
-            long long kk = -1;
-            if (kp < col[o + 1]) {
-              const int o2 = org[kp];
-              kk = (o2 == o) ? k : a.eidx[tri_index(j, o2)];
-              if (kk >= 0 && kk != k && !a.gnz[kk]) kk = -1;
-            }
-            unsigned act = __ballot_sync(0xffffffffu, kk >= 0);
-            while (act) {
-              const int l = __ffs(act) - 1;
-              act &= act - 1;
-              const long long kq = __shfl_sync(0xffffffffu, kk, l);
-              const uint32_t* P = a.ws.bits + (size_t)(kb + l) * W;
-              const uint32_t* GK = G + (size_t)kq * W;
-              for (int w = lane; w < W; w += 32) {
-                uint32_t m = P[w] & g.any_nt[w] & shr1_word(GK, w, W);
-                while (m) {
-                  const int bb = __ffs(m) - 1;
-                  m &= m - 1;
-                  const int Bn = g.item_next[(w << 5) + bb] - g.T;
-                  atomicOr(&bset[Bn >> 5], 1u << (Bn & 31));
-                }
+        uint32_t r[KW], bits[KW];
+#pragma unroll
+        for (int i = 0; i < KW; ++i) {
+          const int w = lane + 32 * i;
+          r[i] = (w < W) ? Gk[w] : 0u;
+          bits[i] = (w < W) ? bp[w] : 0u;
+        }
+        bool any_change = false;
+        for (int round = 0; round < 64 * kWMaxW; ++round) {
+          // the self entry's waiting items whose advance is good at (j, o)
+          if (self) {
+#pragma unroll
+            for (int i = 0; i < KW; ++i) {
+              if (32 * i >= W) break;
+              const int w = lane + 32 * i;
+              uint32_t nxt = __shfl_down_sync(0xffffffffu, r[i], 1);
+              const uint32_t wrap = (i + 1 < KW) ? __shfl_sync(0xffffffffu, r[i + 1], 0) : 0u;
+              if (lane == 31) nxt = wrap;
+              const uint32_t sh1 = (r[i] >> 1) | (nxt << 31);
+              uint32_t m = (w < W) ? (E[w] & s_expn[w] & sh1) : 0u;
+              while (m) {
+                const int bb = __ffs(m) - 1;
+                m &= m - 1;
+                const int Bn = tb.item_next[(w << 5) + bb] - g.T;
+                const uint32_t bit = 1u << (Bn & 31);
+                if (!(s_bset[Bn >> 5] & bit)) atomicOr(&s_bset[Bn >> 5], bit);
               }
             }
+            __syncwarp();
           }
-          __syncwarp();
+          // complete items whose left side is turned good
           bool ch = false;
-          for (int w = lane; w < W; w += 32) {
-            uint32_t add = 0;
-            uint32_t m = bits[w] & g.complete[w];
+#pragma unroll
+          for (int i = 0; i < KW; ++i) {
+            const int w = lane + 32 * i;
+            uint32_t m = (w < W) ? (bits[i] & tb.complete[w] & ~r[i]) : 0u;
             while (m) {
               const int bb = __ffs(m) - 1;
               m &= m - 1;
-              const int L2 = g.item_lhs[(w << 5) + bb];
-              if ((bset[L2 >> 5] >> (L2 & 31)) & 1u) add |= 1u << bb;
-            }
-            const uint32_t s = shr1_word(Gk, w, W);
-            if (gap) add |= g.next_any[w] & s;
-            if (self_si >= 0) add |= a.expn[(size_t)self_si * W + w] & s;
-            add &= bits[w];
-            const uint32_t old = Gk[w];
-            if ((old | add) != old) {
-              Gk[w] = old | add;
-              ch = true;
+              const int L2 = tb.item_lhs[(w << 5) + bb];
+              if ((s_bset[L2 >> 5] >> (L2 & 31)) & 1u) {
+                r[i] |= 1u << bb;
+                ch = true;
+              }
             }
           }
           if (!__any_sync(0xffffffffu, ch)) break;
-          changed = true;
-          if (lane == 0) a.gnz[k] = 1;
+          any_change = true;
+          good_in_row<KW>(r, bits, inrow, W);
+          if (!self) break;
+        }
+        if (any_change) {
+          bool nz = false;
+#pragma unroll
+          for (int i = 0; i < KW; ++i) {
+            const int w = lane + 32 * i;
+            if (w < W) Gk[w] = r[i];
+            nz |= r[i] != 0;
+          }
+          nz = __any_sync(0xffffffffu, nz);
+          if (lane == 0 && nz) a.gnz[k] = 1;
         }
       }
-      if (changed && lane == 0) s_flag = 1;
       __syncthreads();
-      const int more = s_flag;
-      __syncthreads();
-      if (!more) break;
     }
+  }
+  __syncthreads();
   }
 }
 
 
 void launch_good(dim3 grid, cudaStream_t st, const DevGrammar& g, int B, const SeqPack& sp) {
-  k_good<<<grid, 32 * kGoodWarps, 0, st>>>(g, B, sp);
+  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps);
+  cudaFuncSetAttribute(k_good, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+  k_good<<<grid, 32 * kGoodWarps, dyn, st>>>(g, B, sp);
 }
 
 int good_warps() { return kGoodWarps; }

@@ -34,7 +34,7 @@ struct SeqPack {
   __host__ __device__ static size_t r(size_t b) { return (b + 255) & ~(size_t)255; }
   __host__ __device__ size_t bytes() const {
     size_t nm = nmax;
-    return r(nm * W * 4) + r(nm * VW * 4) + r((nm + 1) * 4) + 6 * r(kWMaxQ * 4) + r(kWMaxQ * 16) + r(kWMaxQ * 32) +
+    return r(nm * W * 4) + r(nm * VW * 4) + r((nm + 1) * 4) + 7 * r(kWMaxQ * 4) + r(kWMaxQ * 16) + r(kWMaxQ * 32) +
            r(nm * 8) + r((size_t)emax * 4) + r((size_t)emax * 8) + r((size_t)emax * W * 4)  // WWs
            + r(nm) + 2 * r((size_t)edge_cap * 4) + r((size_t)edge_cap * 32) + 3 * r((size_t)n * 4) +
            r((size_t)emax * VW * 4) + r(32)                                                 // SeqRec
@@ -60,6 +60,7 @@ struct SeqPack {
     a.ws.g_end = (int32_t*)take(kWMaxQ * 4);
     a.ws.g_len = (int32_t*)take(kWMaxQ * 4);
     a.ws.g_last = (int32_t*)take(kWMaxQ * 4);
+    a.ws.key_q = (int32_t*)take(kWMaxQ * 4);
     a.ws.g_tail = (uint32_t*)take(kWMaxQ * 16);
     a.ws.g_lbl = (uint32_t*)take(kWMaxQ * 32);
     a.ws.ssum = (uint32_t*)take(nm * 8);

@@ -50,6 +50,38 @@ struct Walk {
     return x[i];
   }
 
+  // Arrival of group gi into its end node: (source column, label set), the
+  // label set all zero for an epsilon edge.
+  __device__ int arrival_src(int gi) const { return sc.g_len[gi] >= 2 ? sc.g_last[gi] : sc.g_src[gi]; }
+  __device__ uint32_t arrival_lbl(int gi, int w) const {
+    const int len = sc.g_len[gi];
+    if (len == 0) return 0u;
+    if (len == 1) return sc.g_lbl[gi * 8 + w];
+    const int a = sc.g_tail[gi * 16 + len - 2];
+    return (w == (a >> 5)) ? (1u << (a & 31)) : 0u;
+  }
+  // Do end states e1 and e2 receive the same arrivals?  (One thread.)
+  __device__ bool same_arrivals(int e1, int e2, int ng) const {
+    int n1 = 0, n2 = 0;
+    for (int gi = 0; gi < ng; ++gi) {
+      n1 += sc.g_end[gi] == e1;
+      n2 += sc.g_end[gi] == e2;
+    }
+    if (n1 != n2) return false;
+    for (int gi = 0; gi < ng; ++gi) {
+      if (sc.g_end[gi] != e1) continue;
+      bool found = false;
+      for (int gj = 0; gj < ng && !found; ++gj) {
+        if (sc.g_end[gj] != e2 || arrival_src(gj) != arrival_src(gi)) continue;
+        bool same = (sc.g_len[gi] == 0) == (sc.g_len[gj] == 0);
+        for (int w = 0; w < 8; ++w) same &= arrival_lbl(gi, w) == arrival_lbl(gj, w);
+        found = same;
+      }
+      if (!found) return false;
+    }
+    return true;
+  }
+
   // One token of a span: frontier (f_q lexer state, f_c column)[0..nf) ->
   // new frontier.  Lexings from the same column with the same end state and
   // the same terminals after the first share one path whose first edge
@@ -102,10 +134,33 @@ struct Walk {
     }
     __syncthreads();
     int ng = sh.ng;
-    // the run up to its last terminal (intermediate nodes)
+    // the run up to its last terminal (intermediate nodes); groups with the
+    // same source, first-terminal set and terminals before the last one
+    // spell the same paths up to it, so they share one chain of nodes
     for (int gi = 0; gi < ng; ++gi) {
       int len = sc.g_len[gi];
       int cur = sc.g_src[gi];
+      if (len >= 2) {
+        if (threadIdx.x == 0) {
+          int share = -1;
+          for (int gj = 0; gj < gi && share < 0; ++gj) {
+            if (sc.g_len[gj] != len || sc.g_src[gj] != cur) continue;
+            bool same = true;
+            for (int w = 0; w < 8; ++w) same &= sc.g_lbl[gj * 8 + w] == sc.g_lbl[gi * 8 + w];
+            for (int t = 0; t + 2 < len; ++t) same &= sc.g_tail[gj * 16 + t] == sc.g_tail[gi * 16 + t];
+            if (same) share = gj;
+          }
+          sh.scratch_i[0] = share;
+        }
+        __syncthreads();
+        const int share = sh.scratch_i[0];
+        __syncthreads();
+        if (share >= 0) {
+          if (threadIdx.x == 0) sc.g_last[gi] = sc.g_last[share];
+          __syncthreads();
+          continue;
+        }
+      }
       for (int t = 0; t + 1 < len; ++t) {
         int c = cols.open_column();
         __syncthreads();
@@ -144,7 +199,38 @@ struct Walk {
     }
     __syncthreads();
     int nt = sh.nt;
+    // end nodes with the same arrivals (sources and labels) have the same
+    // incoming paths: one column serves all their lexer states.  Each end's
+    // arrivals are hashed (sh.list) and counted (sh.prefix, free until the
+    // nodes are built); the smallest equal end is its representative.
+    for (int ti = threadIdx.x; ti < nt; ti += blockDim.x) {
+      const int e = sc.f_q[ti];
+      uint32_t h = 0;
+      int cnt = 0;
+      for (int gi = 0; gi < ng; ++gi) {
+        if (sc.g_end[gi] != e) continue;
+        uint32_t x = (uint32_t)arrival_src(gi) * 0x9E3779B1u + (sc.g_len[gi] == 0 ? 0x85EBCA6Bu : 0u);
+        for (int w = 0; w < 8; ++w) x = (x ^ arrival_lbl(gi, w)) * 0xC2B2AE35u + (uint32_t)w;
+        h += x ^ (x >> 16);
+        ++cnt;
+      }
+      sh.list[ti] = (int32_t)h;
+      sh.prefix[ti] = cnt;
+    }
+    __syncthreads();
+    for (int ti = threadIdx.x; ti < nt; ti += blockDim.x) {
+      int rep = ti;
+      for (int tj = 0; tj < ti; ++tj)
+        if (sh.list[tj] == sh.list[ti] && sh.prefix[tj] == sh.prefix[ti] &&
+            same_arrivals(sc.f_q[ti], sc.f_q[tj], ng)) {
+          rep = tj;
+          break;
+        }
+      sc.key_q[ti] = rep;
+    }
+    __syncthreads();
     for (int ti = 0; ti < nt; ++ti) {
+      if (sc.key_q[ti] != ti) continue;
       int e = sc.f_q[ti];
       int c = cols.open_column();
       __syncthreads();
@@ -169,6 +255,8 @@ struct Walk {
       __syncthreads();
     }
     if (threadIdx.x == 0) {
+      for (int ti = 0; ti < nt; ++ti)
+        if (sc.key_q[ti] != ti) sc.f_c[ti] = sc.f_c[sc.key_q[ti]];
       int k = 0;
       for (int ti = 0; ti < nt; ++ti)
         if (!cols.column_empty(sc.f_c[ti])) {

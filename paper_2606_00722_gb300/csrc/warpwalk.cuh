@@ -39,6 +39,7 @@ struct WWs {  // per-warp global workspace
   int32_t* g_end;    // [kWMaxQ]
   int32_t* g_len;    // [kWMaxQ]
   int32_t* g_last;   // [kWMaxQ]
+  int32_t* key_q;    // [kWMaxQ]  representative of each end node (span step)
   uint32_t* g_tail;  // [kWMaxQ][4]  terminals 1..12 packed 4 per word
   uint32_t* g_lbl;   // [kWMaxQ][8]  first-terminal label set
 };
@@ -65,6 +66,7 @@ struct WSh {  // per-warp shared memory
   uint32_t touched[kWCols / 32];
   uint32_t dirty[kWCols / 32];
   uint32_t vset[kWMaxVW], vdone[kWMaxVW], nt[kWMaxVW];
+  uint32_t vdone_tot[kWMaxVW];  // nonterminals newly completed from the origin being closed
   uint32_t lbl[kWMaxW];
   uint32_t expn[kWMaxW];
 };
@@ -418,9 +420,9 @@ class WarpWalker {
   // column have distinct origins, so lanes never share a destination row.
   // `which` selects the summary filter (0: waited nonterminals, 1: expected
   // terminals, -1: none) tested against `fold`.
-  __device__ void scatter(int col, const uint32_t* M, bool shift, int which, uint32_t fold) {
+  __device__ void scatter(int col, const uint32_t* M, bool shift, int which, uint32_t fold, int skip_org = -1) {
     const int lane = wl_lane();
-    const long long b = cbeg(col), e = cend(col);
+    const long long b = cbeg(col), e = skip_org >= 0 ? cend(col) - 1 : cend(col);
     if (!SM && W > 16) {  // wide rows in the global stage: the lanes share each entry's words
       for (long long base = b; base < e; base += 32) {
         const long long k = base + lane;
@@ -541,6 +543,39 @@ class WarpWalker {
     }
   }
 
+  // row |= shift(items of E waiting on a member of the nonterminal set nts);
+  // returns whether row changed
+  __device__ bool row_into_waiting(uint32_t* row, const uint32_t* E, const uint32_t* nts) {
+    bool ch = false;
+    uint32_t carry = 0;
+    for (int base = 0; base < W; base += 32) {
+      const int w = base + wl_lane();
+      uint32_t x = 0;
+      if (w < W) {
+        uint32_t m = E[w] & g.any_nt[w];
+        while (m) {
+          const int b = __ffs(m) - 1;
+          m &= m - 1;
+          const int B = g.item_next[(w << 5) + b] - g.T;
+          if ((nts[B >> 5] >> (B & 31)) & 1u) x |= 1u << b;
+        }
+      }
+      uint32_t prev = __shfl_up_sync(0xffffffffu, x, 1);
+      if (wl_lane() == 0) prev = carry;
+      carry = __shfl_sync(0xffffffffu, x, 31);
+      const uint32_t add = (x << 1) | (prev >> 31);
+      if (w < W && add) {
+        const uint32_t old = row[w];
+        if ((old | add) != old) {
+          row[w] = old | add;
+          ch = true;
+        }
+      }
+    }
+    __syncwarp();
+    return __any_sync(0xffffffffu, ch);
+  }
+
   // ------------------------------------------------------------ columns
   __device__ int open_column() {
     if (ncols >= nmax) {
@@ -648,35 +683,56 @@ class WarpWalker {
       if (wl_lane() == 0) sh.dirty[o >> 5] &= ~(1u << (o & 31));
       __syncwarp();
       uint32_t* row = row_of(o);
-      PH_BEGIN(t_row);
-      row_advance(row, gap ? g.next_any : g.nullable_next);
-      PH_END(3, t_row);
-      PH_BEGIN(t_nts);
-      row_scan(row, sh.vset, sum_of(o));
-      if (o == c) continue;  // completions from c at c: nullable / gap rules above
-      for (int v = wl_lane(); v < VW; v += 32) sh.nt[v] = 0;
-      __syncwarp();
-      row_nts(row, g.complete, true, sh.nt);
-      bool any = false;
-      uint32_t* bd = bdone_of(o);
-      for (int v = wl_lane(); v < VW; v += 32) {
-        uint32_t d = sh.nt[v] & ~bd[v];
-        sh.nt[v] = d;
-        any |= d != 0;
-        bd[v] |= d;
+      if (o == c) {  // completions from c at c: the nullable / gap advance rules
+        PH_BEGIN(t_row);
+        row_advance(row, gap ? g.next_any : g.nullable_next);
+        PH_END(3, t_row);
+        row_scan(row, sh.vset, sum_of(o));
+        continue;
       }
-      __syncwarp();
-      PH_END(4, t_nts);
-      if (!__any_sync(0xffffffffu, any)) continue;
+      // Completions from o advance the items of column o; of those, only the
+      // entry with origin o itself (the last one: entries are stored by
+      // ascending origin) feeds row o again.  Close that loop first, then
+      // scatter everything completed from o once over the other entries.
+      const long long ke = cend(o);
+      const bool self = ke > cbeg(o) && eorg(ke - 1) == o;
+      uint32_t* bd = bdone_of(o);
+      for (int v = wl_lane(); v < VW; v += 32) sh.vdone_tot[v] = 0;
+      bool any_tot = false;
+      for (int round = 0; round < 64 * kWMaxW; ++round) {
+        PH_BEGIN(t_row);
+        row_advance(row, gap ? g.next_any : g.nullable_next);
+        PH_END(3, t_row);
+        PH_BEGIN(t_nts);
+        for (int v = wl_lane(); v < VW; v += 32) sh.nt[v] = 0;
+        __syncwarp();
+        row_nts(row, g.complete, true, sh.nt);
+        bool any = false;
+        for (int v = wl_lane(); v < VW; v += 32) {
+          const uint32_t d = sh.nt[v] & ~bd[v];
+          sh.nt[v] = d;
+          any |= d != 0;
+          bd[v] |= d;
+          sh.vdone_tot[v] |= d;
+        }
+        __syncwarp();
+        PH_END(4, t_nts);
+        any = __any_sync(0xffffffffu, any);
+        any_tot |= any;
+        if (!any || !self) break;
+        if (!row_into_waiting(row, ebits(ke - 1), sh.nt)) break;
+      }
+      row_scan(row, sh.vset, sum_of(o));
+      if (!any_tot) continue;
       PH_BEGIN(t_expn);
-      // EXPN: items waiting on a newly completed nonterminal
-      expn_of_set(g, sh.nt, sh.expn);
+      // EXPN: items waiting on a nonterminal newly completed from o
+      expn_of_set(g, sh.vdone_tot, sh.expn);
       __syncwarp();
       PH_END(5, t_expn);
       PH_BEGIN(t_part);
       uint32_t fold = 0;
-      for (int v = 0; v < VW; ++v) fold |= sh.nt[v];
-      scatter(o, sh.expn, true, 0, fold);
+      for (int v = 0; v < VW; ++v) fold |= sh.vdone_tot[v];
+      scatter(o, sh.expn, true, 0, fold, self ? o : -1);
       if (status) return;
       PH_END(6, t_part);
     }
@@ -883,10 +939,28 @@ class WarpWalker {
       __syncwarp();
     }
     PH_END(0, t_group);
-    // intermediate nodes: the run up to its last terminal
+    // intermediate nodes: the run up to its last terminal; groups with the
+    // same source, first-terminal set and terminals before the last one
+    // spell the same paths up to it, so they share one chain of nodes
     for (int gi = 0; gi < ng; ++gi) {
       int len = ws.g_len[gi];
       int cur = ws.g_src[gi];
+      if (len >= 2) {
+        int share = -1;
+        for (int gb = 0; gb < gi && share < 0; gb += 32) {
+          const int gj = gb + (int)wl_lane();
+          bool same = gj < gi && ws.g_len[gj] == len && ws.g_src[gj] == cur;
+          for (int w = 0; w < 8 && same; ++w) same = ws.g_lbl[gj * 8 + w] == ws.g_lbl[gi * 8 + w];
+          for (int t = 1; t + 1 < len && same; ++t) same = tail_term(gj, t) == tail_term(gi, t);
+          const unsigned m = __ballot_sync(0xffffffffu, same);
+          if (m) share = gb + __ffs(m) - 1;
+        }
+        if (share >= 0) {
+          if (wl_lane() == 0) ws.g_last[gi] = ws.g_last[share];
+          __syncwarp();
+          continue;
+        }
+      }
       for (int t = 0; t + 1 < len; ++t) {
         if (t == 0) {
           label_set(ws.g_lbl + gi * 8);
@@ -901,7 +975,7 @@ class WarpWalker {
       if (wl_lane() == 0) ws.g_last[gi] = cur;
       __syncwarp();
     }
-    // one node per distinct end state, ascending
+    // the distinct end states, ascending (the old frontier is consumed)
     int nt = 0;
     int prev = -1;
     for (;;) {
@@ -912,6 +986,30 @@ class WarpWalker {
       }
       for (int off = 16; off; off >>= 1) best = min(best, __shfl_xor_sync(0xffffffffu, best, off));
       if (best == 0x7fffffff) break;
+      if (wl_lane() == 0) ws.f_q[nt] = best;
+      ++nt;
+      prev = best;
+    }
+    __syncwarp();
+    // end nodes with the same arrivals (sources and labels) have the same
+    // incoming paths: one column serves all their lexer states; the smallest
+    // equal end is the representative (ws.f_c holds a hash of the arrivals
+    // until the columns are made)
+    for (int ti = wl_lane(); ti < nt; ti += 32) ws.f_c[ti] = (int32_t)arrivals_hash(ws.f_q[ti], ng);
+    __syncwarp();
+    for (int ti = wl_lane(); ti < nt; ti += 32) {
+      int rep = ti;
+      for (int tj = 0; tj < ti; ++tj)
+        if (ws.f_c[tj] == ws.f_c[ti] && same_arrivals(ws.f_q[ti], ws.f_q[tj], ng)) {
+          rep = tj;
+          break;
+        }
+      ws.key_q[ti] = rep;
+    }
+    __syncwarp();
+    for (int ti = 0; ti < nt; ++ti) {
+      if (ws.key_q[ti] != ti) continue;
+      const int best = ws.f_q[ti];
       int c = open_column();
       if (c < 0) return false;
       for (int gi = 0; gi < ng; ++gi) {
@@ -923,25 +1021,78 @@ class WarpWalker {
           label_set(ws.g_lbl + gi * 8);
           arrive(ws.g_src[gi], sh.lbl, true);
         } else {
-          uint32_t tw = ws.g_tail[gi * 4 + ((len - 2) >> 2)];
-          label_one((tw >> (8 * ((len - 2) & 3))) & 0xff);
+          label_one(tail_term(gi, len - 1));
           arrive(ws.g_last[gi], sh.lbl, true);
         }
       }
       close_column(c, false);
       finish_column(c);
       if (status) return false;
-      if (!column_empty(c)) {
-        if (wl_lane() == 0) {
-          ws.f_q[nt] = best;
-          ws.f_c[nt] = c;
-        }
-        ++nt;
+      if (wl_lane() == 0) ws.f_c[ti] = c;
+      __syncwarp();
+    }
+    // the new frontier: (end state, column) of the non-empty columns
+    for (int ti = wl_lane(); ti < nt; ti += 32)
+      if (ws.key_q[ti] != ti) ws.f_c[ti] = ws.f_c[ws.key_q[ti]];  // representatives are columns by now
+    __syncwarp();
+    int nk = 0;
+    for (int ti = 0; ti < nt; ++ti) {
+      const int c = ws.f_c[ti];
+      if (column_empty(c)) continue;
+      if (wl_lane() == 0) {
+        ws.f_q[nk] = ws.f_q[ti];
+        ws.f_c[nk] = c;
       }
       __syncwarp();
-      prev = best;
+      ++nk;
     }
-    nf = nt;
+    nf = nk;
+    return true;
+  }
+
+  // terminal t (1 .. len-1) of group gi's run
+  __device__ int tail_term(int gi, int t) const {
+    return (ws.g_tail[gi * 4 + ((t - 1) >> 2)] >> (8 * ((t - 1) & 3))) & 0xff;
+  }
+  // arrival of group gi into its end node: source column and label set (all
+  // zero: epsilon)
+  __device__ int arrival_src(int gi) const { return ws.g_len[gi] >= 2 ? ws.g_last[gi] : ws.g_src[gi]; }
+  __device__ uint32_t arrival_lbl(int gi, int w) const {
+    const int len = ws.g_len[gi];
+    if (len == 0) return 0u;
+    if (len == 1) return ws.g_lbl[gi * 8 + w];
+    const int a = tail_term(gi, len - 1);
+    return (w == (a >> 5)) ? (1u << (a & 31)) : 0u;
+  }
+  __device__ uint32_t arrivals_hash(int e, int ng) const {
+    uint32_t h = 0;
+    for (int gi = 0; gi < ng; ++gi) {
+      if (ws.g_end[gi] != e) continue;
+      uint32_t x = (uint32_t)arrival_src(gi) * 0x9E3779B1u + (ws.g_len[gi] == 0 ? 0x85EBCA6Bu : 0u);
+      for (int w = 0; w < 8; ++w) x = (x ^ arrival_lbl(gi, w)) * 0xC2B2AE35u + (uint32_t)w;
+      h += x ^ (x >> 16);
+    }
+    return h;
+  }
+  // do end states e1 and e2 receive the same arrivals?  (one lane)
+  __device__ bool same_arrivals(int e1, int e2, int ng) const {
+    int n1 = 0, n2 = 0;
+    for (int gi = 0; gi < ng; ++gi) {
+      n1 += ws.g_end[gi] == e1;
+      n2 += ws.g_end[gi] == e2;
+    }
+    if (n1 != n2) return false;
+    for (int gi = 0; gi < ng; ++gi) {
+      if (ws.g_end[gi] != e1) continue;
+      bool found = false;
+      for (int gj = 0; gj < ng && !found; ++gj) {
+        if (ws.g_end[gj] != e2 || arrival_src(gj) != arrival_src(gi)) continue;
+        bool same = (ws.g_len[gi] == 0) == (ws.g_len[gj] == 0);
+        for (int w = 0; w < 8; ++w) same &= arrival_lbl(gi, w) == arrival_lbl(gj, w);
+        found = same;
+      }
+      if (!found) return false;
+    }
     return true;
   }
 

@@ -18,11 +18,11 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 # translation units, compiled in parallel and linked into one library
 _SRC = [os.path.join(_HERE, 'csrc', f) for f in
         ('epic.cu', 'kernels_walk.cu', 'kernels_select.cu', 'region_forward.cu', 'region_good.cu',
-         'region_check_sm.cu', 'region_check_global.cu', 'grammar.cpp')]
+         'region_check_sm.cu', 'region_check_global.cu', 'peak.cu', 'grammar.cpp')]
 _DEPS = _SRC + [os.path.join(_HERE, 'csrc', f) for f in
                 ('grammar.h', 'device.cuh', 'walk.cuh', 'cover.cuh', 'skeleton.cuh', 'warpwalk.cuh', 'packs.cuh',
-                 'seqpack.cuh', 'launch.h', 'region.cuh', 'region_check.cuh')] + \
-    [os.path.join(_HERE, '..', 'include', 'epic.h')]
+                 'seqpack.cuh', 'launch.h', 'region.cuh', 'region_check.cuh', 'gscols.cuh')] + \
+    [os.path.join(_HERE, '..', 'include', 'epic.h'), os.path.join(_HERE, '..', 'include', 'epic_measure.h')]
 LIB_PATH = os.path.join(_HERE, '_build', 'libepic.so')
 ARCH_FLAGS = ['-gencode', 'arch=compute_103a,code=sm_103a']
 COMPILE_FLAGS = ARCH_FLAGS + ['-lineinfo', '-O3', '-std=c++17', '-Xcompiler', '-fPIC']
@@ -87,7 +87,7 @@ EXPORTS = ('epic_grammar_create', 'epic_grammar_destroy', 'epic_grammar_lexer_st
            'epic_lexer_table_build', 'epic_lexer_table_destroy', 'epic_lexer_table_copy',
            'epic_validate_batch', 'epic_validate_batch_noalloc',
            'epic_pick_candidates', 'epic_select_compatible_subset', 'epic_commit',
-           'epic_get_stats', 'epic_status_string')
+           'epic_get_stats', 'epic_status_string', 'epic_measure_int_peak', 'epic_last_kernel_times')
 
 
 def load(path: str | None = None):
@@ -112,6 +112,10 @@ def load(path: str | None = None):
     lib.epic_select_compatible_subset.argtypes = [vp, vp, vp, i32, i32, vp, i32, vp, vp, vp, vp]
     lib.epic_commit.argtypes = [vp, i32, i32, vp, i32, vp, vp, vp]
     lib.epic_get_stats.argtypes = [vp, C.POINTER(_Stats), C.c_size_t, C.c_int]
+    lib.epic_measure_int_peak.argtypes = [C.POINTER(C.c_double), C.POINTER(C.c_double), vp]
+    lib.epic_measure_int_peak.restype = C.c_int
+    lib.epic_last_kernel_times.argtypes = [vp, C.POINTER(C.c_float), C.POINTER(C.c_char_p), C.c_int]
+    lib.epic_last_kernel_times.restype = C.c_int
     _lib = lib
     return lib
 
@@ -218,6 +222,16 @@ class LexTable:
         _check(load().epic_get_stats(self.h, C.byref(s), C.sizeof(s), int(reset)), 'epic_get_stats')
         return {n: int(getattr(s, n)) for n, _ in _Stats._fields_}
 
+    def kernel_times(self) -> dict:
+        """epic_last_kernel_times: {kernel name: ms} of the last
+        validate_batch call on this table (synchronizes)."""
+        ms = (C.c_float * 4)()
+        names = (C.c_char_p * 4)()
+        n = load().epic_last_kernel_times(self.h, ms, names, 4)
+        if n < 0:
+            raise EpicError(ERR_CUDA, 'epic_last_kernel_times')
+        return {names[i].decode(): float(ms[i]) for i in range(n)}
+
     def close(self):
         if getattr(self, 'h', None):
             load().epic_lexer_table_destroy(self.h)
@@ -228,6 +242,17 @@ class LexTable:
             self.close()
         except Exception:
             pass
+
+
+def measure_int_peak(stream=None):
+    """epic_measure_int_peak: (word operations per second, kernel ms) of the
+    integer pipe on the current device (the roofline denominator of the
+    walks)."""
+    rate, ms = C.c_double(0), C.c_double(0)
+    r = load().epic_measure_int_peak(C.byref(rate), C.byref(ms), _stream(stream))
+    if r != 0:
+        raise EpicError(r, 'epic_measure_int_peak')
+    return rate.value, ms.value
 
 
 def validate_batch(g: Grammar, t: LexTable, x, pos, cand, valid, stream=None):
