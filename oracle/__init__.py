@@ -3,8 +3,9 @@
 A plain CPU implementation (``epic_oracle.cpp``) of what the hot path
 computes, written from the paper: the completability predicate of Sec. 3,
 the partial-output graph of Alg. 2, the Earley-style graph parser of Alg. 3,
-the flattened regular cover of Sec. 4.3 / App. A.2, and Alg. 4's relaxed
-subset selection with exact shrink.  It shares no code with the CUDA path.
+the flattened regular cover of Sec. 4.3 / App. A.2, Alg. 4's relaxed
+subset selection with exact shrink, and Alg. 1's sequential rejection
+fallback.  It shares no code with the CUDA path.
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and the benchmark's CPU-baseline
 leg may import this module.
@@ -62,6 +63,8 @@ def _load():
             lib.orc_select.argtypes = [C.c_void_p, i32p, C.c_int, C.c_int, i32p, C.c_int, i32p,
                                        f32p, u8p, i64p, i64p]
             lib.orc_commit.argtypes = [i32p, C.c_int, C.c_int, i32p, C.c_int, i32p, u8p]
+            lib.orc_fallback.argtypes = [C.c_void_p, i32p, C.c_int, C.c_int, i32p, C.c_int, i32p, f32p,
+                                         C.c_int, i32p, u8p, i32p, i64p]
             _lib = lib
     return _lib
 
@@ -208,6 +211,31 @@ class Oracle:
             raise ValueError('NaN confidence')
         self.last_select_counts = (nc.value, ne.value)
         return sel
+
+    def fallback(self, x, pos, cand, conf, n_target, selected=None):
+        """Alg. 1's sequential rejection fallback after the selected batch
+        was committed (x already holds it): returns (x updated, filled [B][k]
+        token committed at each slot by the fallback or -1, exact checks)."""
+        x = np.array(x, np.int32, copy=True)
+        pos = np.ascontiguousarray(pos, np.int32)
+        cand = np.ascontiguousarray(cand, np.int32)
+        conf = np.ascontiguousarray(conf, np.float32)
+        n_target = np.ascontiguousarray(n_target, np.int32)
+        B, n = x.shape
+        k = pos.shape[1]
+        K = cand.shape[2]
+        filled = np.full((B, k), -1, np.int32)
+        sel = None if selected is None else np.ascontiguousarray(selected, np.uint8)
+        nchk = C.c_longlong(0)
+        r = self._lib.orc_fallback(self.h, _p(x, C.c_int32), B, n, _p(pos, C.c_int32), k, _p(cand, C.c_int32),
+                                   _p(conf, C.c_float), K, _p(n_target, C.c_int32),
+                                   None if sel is None else _p(sel, C.c_uint8), _p(filled, C.c_int32),
+                                   C.byref(nchk))
+        if r == -1:
+            raise ValueError('a proposed position is out of range')
+        if r == -2:
+            raise ValueError('NaN confidence')
+        return x, filled, nchk.value
 
     @staticmethod
     def commit(x, pos, tok, selected):

@@ -962,6 +962,80 @@ int orc_select(void* h, const int* x, int B, int n, const int* pos, int k, const
   return 0;
 }
 
+// Sequential rejection fallback (Alg. 1, the loop after the selected batch
+// B is committed): for each of the fill[b] = max(0, n_target[b] - |B|)
+// remaining commits, take the highest-confidence candidate (over every
+// proposed position and its K candidates) whose position is still masked and
+// that was not rejected; while x (+) c fails the exact test of Sec. 3, reject
+// it (its logit is suppressed) and take the next; commit the accepted one to
+// x.  Readings: candidates are ordered by descending confidence, then
+// ascending position, then ascending candidate index; positions committed
+// before (by B or earlier in this loop) are not candidates; the loop stops
+// early when no candidate is left.  x is updated in place; filled[b][j] =
+// the token committed at slot j by this loop, else -1; *checks counts exact
+// tests.  selected may be NULL (|B| = 0).  Returns -2 on a NaN confidence
+// (nothing of that sequence is committed), -1 on a position out of range.
+int orc_fallback(void* h, int* x, int B, int n, const int* pos, int k, const int* cand, const float* conf, int K,
+                 const int* n_target, const uint8_t* selected, int* filled, long long* checks) {
+  Oracle* O = (Oracle*)h;
+  Grammar& g = O->g;
+  LexMemo memo;
+  long long nchk = 0;
+  int ret = 0;
+  for (int b = 0; b < B; ++b) {
+    int* xb = x + (long long)b * n;
+    for (int j = 0; j < k; ++j) filled[b * k + j] = -1;
+    int nsel = 0;
+    if (selected)
+      for (int j = 0; j < k; ++j) nsel += selected[b * k + j] == 1;
+    int fill = n_target[b] - nsel;
+    struct Q {
+      int j, c, p, t;
+      float cf;
+    };
+    std::vector<Q> order;
+    bool nan = false;
+    for (int j = 0; j < k; ++j) {
+      int p = pos[b * k + j];
+      if (p < 0 || p >= n) return -1;
+      for (int c = 0; c < K; ++c) {
+        float cf = conf[((long long)b * k + j) * K + c];
+        if (cf != cf) nan = true;
+        order.push_back({j, c, p, cand[((long long)b * k + j) * K + c], cf});
+      }
+    }
+    if (nan) {
+      ret = -2;
+      continue;
+    }
+    std::stable_sort(order.begin(), order.end(), [](const Q& a, const Q& q) {
+      if (a.cf != q.cf) return a.cf > q.cf;
+      if (a.p != q.p) return a.p < q.p;
+      return a.c < q.c;
+    });
+    std::vector<char> rejected(order.size(), 0);
+    for (int r = 0; r < fill; ++r) {
+      bool committed = false;
+      for (size_t q = 0; q < order.size() && !committed; ++q) {
+        if (rejected[q] || xb[order[q].p] >= 0) continue;  // committed positions are not candidates
+        std::vector<int> y(xb, xb + n);
+        y[order[q].p] = order[q].t;
+        ++nchk;
+        if (order[q].t >= 0 && exact_valid(g, y, memo)) {
+          xb[order[q].p] = order[q].t;
+          filled[b * k + order[q].j] = order[q].t;
+          committed = true;
+        } else {
+          rejected[q] = 1;
+        }
+      }
+      if (!committed) break;  // every candidate rejected
+    }
+  }
+  if (checks) *checks = nchk;
+  return ret;
+}
+
 // Commit (Alg. 1): write the selected tokens into x.
 void orc_commit(int* x, int B, int n, const int* pos, int k, const int* tok, const uint8_t* selected) {
   for (int b = 0; b < B; ++b)

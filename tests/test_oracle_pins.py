@@ -650,3 +650,76 @@ def test_cover_valid_brute_force_over_gap_fillings():
             checked += 1
             agree_true += expect
     assert checked > 3000 and 0 < agree_true < checked
+
+
+# ------------------------------------------------------------------ Alg. 1's fallback
+def fallback_python(O, x, pos, cand, conf, fill):
+    """Alg. 1's sequential rejection loop transcribed with the oracle's exact
+    test as the primitive: `fill` times, take the highest-confidence
+    candidate at a still-masked position that was not rejected (ties:
+    position, then candidate index); reject while x (+) c is invalid."""
+    x = x.copy()
+    order = sorted(((-float(conf[j, c]), int(pos[j]), c, j) for j in range(len(pos)) for c in range(cand.shape[1])))
+    rejected = set()
+    filled = {}
+    for _ in range(fill):
+        for (_, p, c, j) in order:
+            if (j, c) in rejected or x[p] >= 0:
+                continue
+            y = x.copy()
+            y[p] = cand[j, c]
+            if O.valid(y):
+                x[p] = cand[j, c]
+                filled[j] = int(cand[j, c])
+                break
+            rejected.add((j, c))
+        else:
+            break
+    return x, filled
+
+
+@pytest.mark.parametrize('name,seed,kw', [('expr-tiny', 42, {}), ('expr-tiny', 44, dict(k=6, K=4)),
+                                          ('json-schema', 42, dict(batch=2, k=6, K=6)),
+                                          ('smiles-256', 43, dict(batch=2, k=6, K=5))])
+def test_fallback_matches_alg1_transcription(name, seed, kw):
+    w = make_workload(name, seed, **kw)
+    O = oracle.Oracle(w.grammar, w.vocab)
+    valid = O.validate_batch(w.x, w.pos, w.cand)
+    tok, conf = oracle.pick_candidates(valid, w.cand, w.conf)
+    sel = O.select(w.x, w.pos, tok, conf)
+    x1 = O.commit(w.x, w.pos, tok, sel)
+    n_target = np.full(w.B, w.k, np.int32)  # fill every proposed position if possible
+    got_x, filled, nchk = O.fallback(x1, w.pos, w.cand, w.conf, n_target, sel)
+    for b in range(w.B):
+        ref_x, ref_f = fallback_python(O, x1[b], w.pos[b], w.cand[b], w.conf[b], int(n_target[b] - sel[b].sum()))
+        np.testing.assert_array_equal(got_x[b], ref_x)
+        assert {j: int(t) for j, t in enumerate(filled[b]) if t >= 0} == ref_f
+    if (n_target - sel.sum(1)).sum() > 0:
+        assert nchk > 0
+
+
+@pytest.mark.parametrize('name,seed', [('expr-tiny', 43), ('json-schema', 45)])
+def test_fallback_invariants(name, seed):
+    """Every fallback commit fills a masked position and keeps the output
+    completable (it was tested with all earlier commits applied); if fewer
+    than asked were committed, every candidate left at a masked position is
+    invalid for the final output (a rejected candidate stays invalid after
+    later commits, by monotonicity of completability, App. D)."""
+    w = make_workload(name, seed, batch=2, k=6, K=6)
+    O = oracle.Oracle(w.grammar, w.vocab)
+    n_target = np.array([3, 6], np.int32)
+    got_x, filled, _ = O.fallback(w.x, w.pos, w.cand, w.conf, n_target)
+    for b in range(w.B):
+        committed = [j for j in range(w.k) if filled[b, j] >= 0]
+        assert len(committed) <= n_target[b]
+        for j in committed:
+            assert w.x[b, w.pos[b, j]] < 0 and got_x[b, w.pos[b, j]] == filled[b, j]
+        assert O.valid(got_x[b]) or not O.valid(w.x[b])
+        if len(committed) < n_target[b]:
+            for j in range(w.k):
+                if got_x[b, w.pos[b, j]] >= 0:
+                    continue
+                for c in range(w.K):
+                    y = got_x[b].copy()
+                    y[w.pos[b, j]] = w.cand[b, j, c]
+                    assert not O.valid(y)
