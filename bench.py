@@ -24,7 +24,15 @@ import numpy as np
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-INT_PEAK_NOTE = '152 SMs x 128 int32 lanes x 2.07 GHz'
+# ncu summaries of the kernels' DRAM traffic (profiles/traffic_<kernel>_<workload>.txt): used only while the
+# kernel's sources hash to the value recorded with the counters
+KERNEL_SOURCES = {
+    'k_validate_warp': ['kernels_walk.cu', 'warpwalk.cuh', 'device.cuh', 'packs.cuh'],
+    'k_forward_gs': ['region_forward.cu', 'gscols.cuh', 'skeleton.cuh', 'walk.cuh', 'device.cuh', 'seqpack.cuh'],
+    'k_forward': ['region_forward.cu', 'warpwalk.cuh', 'device.cuh', 'seqpack.cuh'],
+    'k_good': ['region_good.cu', 'gscols.cuh', 'device.cuh', 'seqpack.cuh'],
+    'k_check': ['region_check.cuh', 'region_check_sm.cu', 'region_check_global.cu', 'warpwalk.cuh', 'device.cuh'],
+}
 
 
 def parse():
@@ -114,12 +122,65 @@ class Clocks:
                 'samples': len(sm)}
 
 
+def kernel_sha(kernel):
+    """Hash of a kernel's source files (tells whether recorded counters still
+    describe the current build)."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES.get(kernel, []):
+        with open(os.path.join(ROOT, 'paper_2606_00722_gb300', 'csrc', f), 'rb') as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel, workload):
+    """DRAM bytes per launch from profiles/traffic_<kernel>_<workload>.txt
+    (key: value lines), or None if absent or recorded for other sources."""
+    path = os.path.join(ROOT, 'profiles', 'traffic_%s_%s.txt' % (kernel, workload))
+    if not os.path.exists(path):
+        return None
+    rec = {}
+    with open(path) as f:
+        for line in f:
+            if ':' in line and not line.startswith('#'):
+                k, v = line.split(':', 1)
+                rec[k.strip()] = v.strip()
+    if rec.get('source_sha16') != kernel_sha(kernel):
+        return None
+    try:
+        return float(rec['dram_bytes_per_launch'])
+    except (KeyError, ValueError):
+        return None
+
+
+def census(workload, batch):
+    """The oracle's chart census of the workload (tests/golden/census_*.json,
+    written by tests/golden/make_census.py): item words per entry, and the
+    (node, origin) pairs of the forward charts of x over the batch (sample
+    mean times the batch) and, where counted, of every check's own chart."""
+    path = os.path.join(ROOT, 'tests', 'golden', 'census_%s.json' % workload)
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        d = json.load(f)
+    per = d.get('per_seq', [])
+    out = {'words': d['words'], 'file': os.path.relpath(path, ROOT)}
+    if per:
+        out['forward_pairs'] = float(np.mean([r['pairs'] for r in per])) * batch
+        out['forward_sample'] = '%d of %d sequences' % (len(per), batch)
+    if 'checks_pairs' in d:
+        out['checks_pairs'] = float(d['checks_pairs'])
+    return out
+
+
 def cpu_baseline(w, seconds):
     """The oracle as it stands on the host cores, on a bounded sample of the
     workload's checks (whole sequences, all their candidates, in order)."""
     import oracle
-    O = oracle.Oracle(w.grammar, w.vocab)
     cores = os.cpu_count() or 1
+    if w.n >= 1024:
+        return cpu_baseline_bounded(w, seconds, cores)
+    O = oracle.Oracle(w.grammar, w.vocab)
     per_seq = w.k * w.K
     t0 = time.perf_counter()
     done = 0
@@ -145,6 +206,47 @@ def cpu_baseline(w, seconds):
             'value_1core': one / dt1,
             'sample_1core': '%d checks of the first sequence, one position per call on 1 thread, %.1f s'
                             % (one, dt1)}
+
+
+def _one_check(args):
+    name, seed, k, b, j, c = args
+    import oracle
+    from synth import make_workload
+    w = make_workload(name, seed, k=k)
+    O = oracle.Oracle(w.grammar, w.vocab)
+    O.validate_batch(w.x[b:b + 1], w.pos[b:b + 1, j:j + 1], w.cand[b:b + 1, j:j + 1, c:c + 1])
+    return 1
+
+
+def cpu_baseline_bounded(w, seconds, cores):
+    """Rows of a thousand tokens: one oracle check takes longer than the whole
+    budget (its chart runs to the end of the row), so one check per core runs
+    for at most `seconds` in worker processes; the rate is the finished checks
+    over the time, or, when none finishes, an upper bound of one check per
+    core over the budget."""
+    import multiprocessing as mp
+    jobs = [(w.name, w.seed, w.k, 0, j % w.k, j // w.k) for j in range(cores)]
+    ctx = mp.get_context('spawn')
+    t0 = time.perf_counter()
+    pool = ctx.Pool(cores)
+    res = [pool.apply_async(_one_check, (a,)) for a in jobs]
+    done = 0
+    deadline = t0 + seconds
+    for r in res:
+        try:
+            done += r.get(timeout=max(0.0, deadline - time.perf_counter()))
+        except mp.TimeoutError:
+            pass
+    dt = time.perf_counter() - t0
+    pool.terminate()
+    pool.join()
+    bound = done == 0
+    value = (cores if bound else done) / dt
+    return {'value': value, 'unit': 'checks/s', 'cores': cores, 'kind': 'oracle',
+            'bound': 'upper' if bound else None,
+            'sample': '%d checks of sequence 0 (one per core, %d positions) for at most %.0f s: %d finished%s'
+                      % (cores, min(cores, w.k), seconds, done,
+                         '; value is one check per core over the budget, an upper bound' if bound else '')}
 
 
 def run_reference(args):
@@ -228,6 +330,7 @@ def main():
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
+    kern = {}  # kernel -> per-step ms (CUDA events around each launch, on this stream)
     with Clocks(local) as clk:
         for i in range(args.steps):
             x.copy_(x0)
@@ -239,6 +342,8 @@ def main():
             epic.select_compatible_subset(g, t, x, pos, tok, conf, sel)
             epic.commit(x, pos, tok, sel)
             ev[i][2].record(stream)
+            for kname, kms in t.kernel_times().items():  # waits for this step's kernels
+                kern.setdefault(kname, []).append(kms)
         torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
@@ -249,7 +354,7 @@ def main():
     # kernels of the timed region: validate's own (one walk kernel, or the
     # forward chart, good masks and region checks) + pick + two selection
     # kernels + commit
-    launches = st['validate_kernels'] + 4 * args.steps
+    launches = st['validate_kernels'] + 4 * args.steps  # + pick, select_spec, select, commit
     ms = float(np.mean(step_ms))
     vms = float(np.mean(val_ms))
     if world > 1:
@@ -283,21 +388,36 @@ def main():
     e2e_step = float(np.mean(e2e_ms))
     h2d = w.x.nbytes + w.pos.nbytes + w.cand.nbytes + w.conf.nbytes
     d2h = w.cand.size + w.pos.size + w.x.nbytes
-    # ---- roofline of the dominant kernel (k_validate): bit-parallel Earley
-    # word operations, 3 passes (predict, scan, complete) over every stored
-    # (node, origin) entry of W words per check
-    pk, pk_kind = peaks()
-    sm_max = pk.get('sm_max_mhz', 2070.0)
-    int_peak = 152 * 128 * sm_max * 1e6 / 1e12  # T word-ops/s
-    entries = st['entries']
-    word_ops = 3.0 * entries * g_words(g)
-    achieved = word_ops / (vms / 1e3) / 1e12 / max(1, args.steps)
-    roof = {'bound': 'alu', 'achieved': achieved, 'peak': int_peak, 'unit': 'T word-ops/s',
-            'frac': achieved / int_peak, 'traffic': None,
-            'peak_source': 'derived: %s (%s sm_max_mhz)' % (INT_PEAK_NOTE, pk_kind),
-            'kernel': ('k_forward + k_good + k_check (epic_validate_batch, by region)' if region
-                       else 'k_validate_warp'),
-            'kernel_ms': vms}
+    # ---- roofline of the dominant kernel of epic_validate_batch: bit-parallel
+    # Earley word operations, 3 passes (predict, scan, complete) over every
+    # (node, origin) pair of the chart the kernel builds, ceil(D / 32) words
+    # each, with the pairs counted by the oracle (tests/golden/census_*.json)
+    # and the kernel's own launch time from CUDA events on this stream
+    kms = {kname: float(np.mean(v)) for kname, v in kern.items()}
+    vkern = {kname: v for kname, v in kms.items() if not kname.startswith('k_select')}
+    dom = max(vkern, key=vkern.get) if vkern else None
+    cen = census(args.workload, w.B)
+    peak_ops, peak_ms = epic.measure_int_peak()
+    peak_t = peak_ops / 1e12
+    work = None
+    if cen and dom in ('k_forward_gs', 'k_forward', 'k_good') and 'forward_pairs' in cen:
+        work = 3.0 * cen['forward_pairs'] * cen['words']
+        work_note = 'forward charts of x: %.0f (node, origin) pairs x %d words x 3 (oracle census, %s)' % (
+            cen['forward_pairs'], cen['words'], cen['forward_sample'])
+    elif cen and dom == 'k_validate_warp' and 'checks_pairs' in cen:
+        work = 3.0 * cen['checks_pairs'] * cen['words']
+        work_note = 'charts of every check: %.0f (node, origin) pairs x %d words x 3 (oracle census)' % (
+            cen['checks_pairs'], cen['words'])
+    else:
+        work_note = 'no oracle census for %s on this workload' % dom
+    achieved = (work / (kms[dom] / 1e3) / 1e12) if (work and dom) else None
+    traffic = recorded_traffic(dom, args.workload) if dom else None
+    roof = {'bound': 'alu', 'achieved': achieved, 'peak': peak_t, 'unit': 'T word-ops/s',
+            'frac': (achieved / peak_t) if achieved else None, 'traffic': traffic,
+            'peak_source': 'measured live: LOP3 + SHF microbenchmark (epic_measure_int_peak, %.2f ms)' % peak_ms,
+            'kernel': dom, 'kernel_ms': kms.get(dom), 'work': work_note,
+            'kernel_share_of_step': (kms[dom] / ms) if dom else None,
+            'kernels_ms': {kname: round(v, 3) for kname, v in kms.items()}}
     line = {'metric': 'candidate validity checks/sec', 'value': value, 'unit': 'checks/s',
             'n_gpus': world, 'steps': args.steps, 'warmup': args.warmup, 'ms_per_step': ms,
             'higher_is_better': True, 'scaling': 'weak', 'vs_baseline': None, 'dtype': 'int32',
@@ -333,13 +453,6 @@ def job_value(checks_per_rank, world, ms):
     """Whole-job throughput: the checks all ranks processed over the slowest
     rank's step time."""
     return checks_per_rank * world / (ms / 1e3)
-
-
-def g_words(g):
-    """Item words per chart entry of the grammar (W = ceil(D / 32))."""
-    spec = g.spec
-    D = sum(len(r) + 1 for _, r in spec.productions) + 2
-    return (D + 31) // 32
 
 
 if __name__ == '__main__':

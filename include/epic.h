@@ -220,6 +220,33 @@ epic_status epic_select_compatible_subset(const epic_grammar* g, const epic_lexe
 epic_status epic_commit(int32_t* d_x, int32_t B, int32_t n, const int32_t* d_pos, int32_t k,
                         const int32_t* d_tok, const uint8_t* d_selected, void* cuda_stream);
 
+/*
+ * Sequential rejection fallback (Alg. 1, the loop that follows the commit of
+ * the selected batch B, "if verification fails or commits remain"): for each
+ * of the max(0, d_n_target[b] - |B_b|) commits still wanted, take the
+ * highest-confidence candidate over every proposed position and its K
+ * candidates whose position is still masked in d_x and that was not
+ * rejected; while x (+) c fails the exact test of Sec. 3, reject it (its
+ * logit is suppressed) and take the next; commit the accepted one.  Ties in
+ * confidence go to the lower position, then the lower candidate index; the
+ * loop ends early when every candidate is rejected.
+ * d_x [B][n] int32, updated in place (call after epic_commit of the selected
+ * batch); d_pos [B][k], d_cand [B][k][K], d_cand_conf [B][k][K] float32 as
+ * for epic_pick_candidates; d_n_target [B] int32 = n_t, the commits wanted
+ * in this step; d_selected [B][k] (1 = in B) or NULL for |B| = 0; output
+ * d_filled [B][k] int32: the token this call committed at slot j, else -1.
+ * One CTA per sequence; each test is a whole-graph walk of x (+) c.
+ * Errors: EPIC_ERR_INVALID_ARG (NULL pointers, sizes < 0),
+ * EPIC_ERR_CAPACITY when k K > 4096.  A NaN confidence or a position out of
+ * range leaves that sequence unchanged (stats.bad_inputs); a test that hits
+ * a capacity limit ends that sequence's loop (stats.overflow).
+ * Asynchronous.
+ */
+epic_status epic_fallback_commit(const epic_grammar* g, const epic_lexer_table* t, int32_t* d_x, int32_t B,
+                                 int32_t n, const int32_t* d_pos, int32_t k, const int32_t* d_cand,
+                                 const float* d_cand_conf, int32_t K, const int32_t* d_n_target,
+                                 const uint8_t* d_selected, int32_t* d_filled, void* cuda_stream);
+
 /* Device counters accumulated since the object was created (or reset). */
 typedef struct {
   uint64_t checks;           /* single-candidate validity checks run           */
@@ -234,6 +261,8 @@ typedef struct {
   uint64_t region_checks;    /* of the checks, those answered by region walks
                                 over a per-sequence forward chart            */
   uint64_t validate_kernels; /* kernel launches made by epic_validate_batch*  */
+  uint64_t fallback_checks;  /* exact tests of the rejection fallback         */
+  uint64_t fallback_commits; /* candidates it committed                       */
 } epic_stats;
 
 /* Copy the counters (synchronizes the lexer table's last stream); out_bytes

@@ -30,13 +30,14 @@ int epic_measure_int_peak(double* word_ops_per_s, double* ms, void* cuda_stream)
 /*
  * Durations of the kernels that the last epic_validate_batch call on t
  * launched, in launch order (by region: the forward charts, the good masks,
- * the region checks; otherwise the one whole-graph walk kernel), measured by
- * CUDA events recorded around each launch on the call's stream.  ms[i]
- * receives kernel i's milliseconds and names[i] (names may be NULL) a static
- * kernel name.  Synchronizes on the last event.  Returns the number of
- * kernels written (at most cap), 0 before any call, -1 on a bad argument or
- * a CUDA error.  The table owns the events; epic_validate_batch_noalloc does
- * not record them.
+ * the region checks; otherwise the one whole-graph walk kernel), followed by
+ * the two kernels of the last epic_select_compatible_subset call on t (the
+ * speculative first tests, then Alg. 4), each measured by CUDA events
+ * recorded around its launch on the call's stream.  ms[i] receives kernel
+ * i's milliseconds and names[i] (names may be NULL) a static kernel name.
+ * Synchronizes on the last events.  Returns the number of kernels written
+ * (at most cap), 0 before any call, -1 on a bad argument or a CUDA error.
+ * The table owns the events; epic_validate_batch_noalloc records none.
  */
 int epic_last_kernel_times(const epic_lexer_table* t, float* ms, const char** names, int cap);
 

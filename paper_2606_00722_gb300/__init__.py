@@ -3,4 +3,5 @@ checking of candidate commits under a CFG, relaxed compatible subset
 selection and commit, behind the C-ABI of ``include/epic.h``."""
 from .epic import (Grammar, LexTable, EpicError, build, load, validate_batch,  # noqa: F401
                    validate_batch_noalloc, measure_int_peak,
-                   pick_candidates, select_compatible_subset, commit, LIB_PATH, EXPORTS)
+                   pick_candidates, select_compatible_subset, commit, fallback_commit, decode_step,
+                   LIB_PATH, EXPORTS)

@@ -134,14 +134,18 @@ struct epic_lexer_table {
   cudaEvent_t kev[4] = {nullptr, nullptr, nullptr, nullptr};
   int nk = 0;
   const char* kname[3] = {nullptr, nullptr, nullptr};
+  // the same around the two kernels of the last epic_select_compatible_subset
+  cudaEvent_t sev[3] = {nullptr, nullptr, nullptr};
+  bool sel_timed = false;
 };
 
 namespace {
 // record event i of the table's kernel timing on st (created on first use)
-void mark(epic_lexer_table* t, int i, cudaStream_t st) {
-  if (!t->kev[i] && cudaEventCreate(&t->kev[i]) != cudaSuccess) t->kev[i] = nullptr;
-  if (t->kev[i]) cudaEventRecord(t->kev[i], st);
+void mark_event(cudaEvent_t* e, cudaStream_t st) {
+  if (!*e && cudaEventCreate(e) != cudaSuccess) *e = nullptr;
+  if (*e) cudaEventRecord(*e, st);
 }
+void mark(epic_lexer_table* t, int i, cudaStream_t st) { mark_event(&t->kev[i], st); }
 }  // namespace
 
 namespace {
@@ -165,31 +169,27 @@ int sm_count() {
   return n > 0 ? n : 1;
 }
 
-// Workspace sizing: columns <= 4096 per walk, entries as many as the budget
-// allows for the CTA count.  EPIC_WORKSPACE_MB (default 2048) caps the total.
-epic_status ensure_workspace(epic_lexer_table* t, int want_ctas, cudaStream_t st) {
+// Block-walk workspace of selection and the fallback: every CTA gets room
+// for one whole chart of a row (4,096 columns, 640 n entries, as the
+// per-sequence forward charts; EPIC_ENTRIES_PER_CTA overrides), and as many
+// CTAs as asked run if their workspaces fit EPIC_WORKSPACE_MB (default
+// 32 GiB), else fewer (the kernels loop over their sequences).
+epic_status ensure_workspace(epic_lexer_table* t, int want_ctas, int n, cudaStream_t st) {
   const epic_grammar* g = t->g;
-  size_t budget_mb = 2048;
+  size_t budget_mb = 32768;
   if (const char* e = getenv("EPIC_WORKSPACE_MB")) budget_mb = strtoull(e, nullptr, 10);
   int W = g->dg.W, VW = g->dg.VW, FW = g->dg.FW;
   WsDims d;
   d.nmax = kMaxCols;
-  long long emax_cap = 1ll << 22;
-  if (const char* e = getenv("EPIC_ENTRIES_PER_CTA")) emax_cap = atoll(e);
-  int ctas = std::max(1, want_ctas);
-  size_t budget = budget_mb << 20;
-  for (;;) {
-    WsDims probe = d;
-    probe.emax = 0;
-    size_t fixed = ws_bytes_per_cta(probe, W, VW, FW);
-    long long per_entry = (long long)(W + 1) * 4;
-    long long room = (long long)(budget / ctas) - (long long)fixed;
-    d.emax = std::min<long long>(emax_cap, room / per_entry);
-    if (d.emax >= 4096 || ctas == 1) break;
-    ctas = std::max(1, ctas / 2);
-  }
-  if (d.emax < 64) return EPIC_ERR_OOM;
+  d.emax = std::max<long long>(4096, 640ll * std::max(1, n));
+  if (const char* e = getenv("EPIC_ENTRIES_PER_CTA")) d.emax = std::max<long long>(64, atoll(e));
+  const size_t budget = budget_mb << 20;
   size_t per = ws_bytes_per_cta(d, W, VW, FW);
+  while (per > budget && d.emax > 4096) {  // not even one CTA fits: smaller charts
+    d.emax = d.emax * 3 / 4;
+    per = ws_bytes_per_cta(d, W, VW, FW);
+  }
+  int ctas = (int)std::max<long long>(1, std::min<long long>(std::max(1, want_ctas), (long long)(budget / per)));
   size_t need = per * (size_t)ctas;
   if (t->d_ws && t->ws_bytes >= need && t->dims.nmax == d.nmax && t->dims.emax == d.emax) {
     t->ctas = ctas;
@@ -292,7 +292,7 @@ epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const in
   sp.W = dg.W;
   sp.VW = dg.VW;
   sp.edge_cap = 32 * sp.nmax;
-  sp.emax = 400ll * n;
+  sp.emax = 640ll * n;
   if (const char* e = getenv("EPIC_SEQ_ENTRIES")) sp.emax = atoll(e);
   size_t budget = (size_t)81920 << 20;
   if (const char* e = getenv("EPIC_SEQ_WORKSPACE_MB")) budget = strtoull(e, nullptr, 10) << 20;
@@ -406,13 +406,16 @@ WsPack pack_of(const epic_lexer_table* t) {
 extern "C" {
 
 #ifdef EPIC_PHASE_TIMERS
-// measurement build only: per-phase cycle counters of the warp walker
+// measurement build only: per-phase cycle counters (the walks' and the GS
+// columns' in out16, the good pass's in out16 + 16)
 int epic_debug_phase_read(unsigned long long* out16, int reset) {
   if (cudaDeviceSynchronize() != cudaSuccess) return -1;
   for (int i = 0; i < 16; ++i) out16[i] = 0;
   if (phase_read_walk(out16, reset) != 0 || phase_read_forward(out16, reset) != 0 ||
       phase_read_check_sm(out16, reset) != 0 || phase_read_check_global(out16, reset) != 0)
     return -1;
+  for (int i = 0; i < 16; ++i) out16[16 + i] = 0;
+  if (phase_read_good(out16 + 16, reset) != 0) return -1;
   return 0;
 }
 #endif
@@ -643,6 +646,8 @@ void epic_lexer_table_destroy(epic_lexer_table* t) {
   cudaFree(t->d_counter);
   for (cudaEvent_t e : t->kev)
     if (e) cudaEventDestroy(e);
+  for (cudaEvent_t e : t->sev)
+    if (e) cudaEventDestroy(e);
   delete t;
 }
 
@@ -714,14 +719,23 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
 
 int epic_last_kernel_times(const epic_lexer_table* t, float* ms, const char** names, int cap) {
   if (!t || (!ms && cap > 0) || cap < 0) return -1;
-  const int n = std::min(t->nk, cap);
-  for (int i = 0; i <= t->nk; ++i)
-    if (!t->kev[i]) return -1;
-  if (t->nk == 0) return 0;
-  if (cudaEventSynchronize(t->kev[t->nk]) != cudaSuccess) return -1;
-  for (int i = 0; i < n; ++i) {
-    if (cudaEventElapsedTime(&ms[i], t->kev[i], t->kev[i + 1]) != cudaSuccess) return -1;
-    if (names) names[i] = t->kname[i];
+  int n = 0;
+  if (t->nk > 0) {
+    for (int i = 0; i <= t->nk; ++i)
+      if (!t->kev[i]) return -1;
+    if (cudaEventSynchronize(t->kev[t->nk]) != cudaSuccess) return -1;
+    for (int i = 0; i < t->nk && n < cap; ++i, ++n) {
+      if (cudaEventElapsedTime(&ms[n], t->kev[i], t->kev[i + 1]) != cudaSuccess) return -1;
+      if (names) names[n] = t->kname[i];
+    }
+  }
+  if (t->sel_timed) {
+    static const char* sname[2] = {"k_select_spec", "k_select"};
+    if (cudaEventSynchronize(t->sev[2]) != cudaSuccess) return -1;
+    for (int i = 0; i < 2 && n < cap; ++i, ++n) {
+      if (cudaEventElapsedTime(&ms[n], t->sev[i], t->sev[i + 1]) != cudaSuccess) return -1;
+      if (names) names[n] = sname[i];
+    }
   }
   return n;
 }
@@ -831,7 +845,7 @@ epic_status epic_select_compatible_subset(const epic_grammar* g, const epic_lexe
   if (!d_x || !d_pos || !d_tok || !d_conf || !d_selected || n == 0) return EPIC_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)cuda_stream;
   int want = std::min(2 * B, sm_count() * 2);
-  epic_status s = ensure_workspace(t, want, st);
+  epic_status s = ensure_workspace(t, want, n, st);
   if (s != EPIC_OK) return s;
   if (t->spec_cap < B) {
     if (t->d_spec) {
@@ -843,11 +857,34 @@ epic_status epic_select_compatible_subset(const epic_grammar* g, const epic_lexe
     t->spec_cap = B;
   }
   t->last = st;
+  mark_event(&t->sev[0], st);
   launch_select_spec(std::min(2 * B, t->ctas), st, g->dg, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_tok,
                      t->d_spec, pack_of(t));
+  mark_event(&t->sev[1], st);
   int ctas = std::min(B, t->ctas);
   launch_select(ctas, st, g->dg, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_tok, d_conf, d_selected, pack_of(t),
                 t->d_spec, t->d_stats);
+  mark_event(&t->sev[2], st);
+  t->sel_timed = t->sev[0] && t->sev[1] && t->sev[2];
+  return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
+}
+
+epic_status epic_fallback_commit(const epic_grammar* g, const epic_lexer_table* tc, int32_t* d_x, int32_t B,
+                                 int32_t n, const int32_t* d_pos, int32_t k, const int32_t* d_cand,
+                                 const float* d_cand_conf, int32_t K, const int32_t* d_n_target,
+                                 const uint8_t* d_selected, int32_t* d_filled, void* cuda_stream) {
+  epic_lexer_table* t = const_cast<epic_lexer_table*>(tc);
+  if (!g || !t || t->g != g || B < 0 || n < 0 || k < 0 || K < 0) return EPIC_ERR_INVALID_ARG;
+  if ((long long)B * k == 0) return EPIC_OK;
+  if ((long long)k * K > kMaxFallbackCand) return EPIC_ERR_CAPACITY;
+  if (!d_x || !d_pos || !d_cand || !d_cand_conf || !d_n_target || !d_filled || n == 0 || K == 0)
+    return EPIC_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  epic_status s = ensure_workspace(t, std::min(B, sm_count() * 2), n, st);
+  if (s != EPIC_OK) return s;
+  t->last = st;
+  launch_fallback(std::min(B, t->ctas), st, g->dg, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_cand, d_cand_conf, K,
+                  d_n_target, d_selected, d_filled, pack_of(t), t->d_stats);
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
 }
 
@@ -876,6 +913,8 @@ epic_status epic_get_stats(const epic_lexer_table* t, epic_stats* out, size_t ou
   out->cover_checks = h[S_COVER];
   out->exact_checks = h[S_EXACT];
   out->selected = h[S_SELECTED];
+  out->fallback_checks = h[S_FB_CHECKS];
+  out->fallback_commits = h[S_FB_COMMITS];
   out->region_checks = t->n_region;
   out->validate_kernels = t->n_vkernels;
   if (reset) {

@@ -36,9 +36,9 @@ struct GsShared {
   uint32_t vset[kMaxVW];              // nonterminals waited on in this column
   uint32_t vdone[kMaxVW];             // ... already predicted
   uint32_t uni[kMaxW];                // union of the column's rows (waited nonterminals)
-  uint32_t wnt[kGsMaxWarps][kMaxVW];  // per-warp sets (recording)
   int32_t cur_o;
   int32_t flag;
+  int32_t labelled;  // the open column has a labelled arrival (else only epsilon ones)
 };
 
 // Grammar tables read by the per-item loops, staged in shared memory:
@@ -96,6 +96,7 @@ class EarleyColsGS {
   int W, VW;
   static constexpr bool kRecord = REC;
   const BlockRec* rec = nullptr;
+  uint32_t* wnt = nullptr;  // recording walks: per-warp nonterminal sets [warps][kMaxVW] (shared memory)
 
   __device__ EarleyColsGS(const DevGrammar& g_, const GsTables& t_, const LexEntry* t, Workspace w, WalkScratch s,
                           WsDims d, WalkShared& shared, GsShared& gss)
@@ -120,6 +121,7 @@ class EarleyColsGS {
       gs.vset[v] = 0;
       gs.vdone[v] = 0;
     }
+    if (threadIdx.x == 0) gs.labelled = 0;
     __syncthreads();
   }
 
@@ -214,6 +216,7 @@ class EarleyColsGS {
   // Arrivals: for every entry (o, y) of column src, stage[o] |= shift(y & M).
   __device__ void arrive(int src, const uint32_t* M, bool shift) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = nwarps();
+    if (shift && threadIdx.x == 0) gs.labelled = 1;
     if (REC && threadIdx.x == 0) {
       if (sh.nedges >= rec->edge_cap) {
         sh.status = kWalkOverflow;
@@ -406,35 +409,43 @@ class EarleyColsGS {
       }
       uint32_t* d0 = ws.stage + (size_t)ws.org[kb + e0] * W;
       uint32_t* d1 = ws.stage + (size_t)ws.org[kb + (has1 ? e1 : e0)] * W;
-      bool ch0 = false, ch1 = false;
-      uint32_t c0 = 0, c1 = 0;
+      // the shifted words (item (p, d) -> (p, d + 1)), then every destination
+      // word loaded before any store (no store may alias a pending load)
+      uint32_t a0[KW], a1[KW];
+      {
+        uint32_t c0 = 0, c1 = 0;
+#pragma unroll
+        for (int i = 0; i < KW; ++i) {
+          uint32_t p0 = __shfl_up_sync(0xffffffffu, v0[i], 1);
+          uint32_t p1 = __shfl_up_sync(0xffffffffu, v1[i], 1);
+          if (lane == 0) {
+            p0 = c0;
+            p1 = c1;
+          }
+          c0 = __shfl_sync(0xffffffffu, v0[i], 31);
+          c1 = __shfl_sync(0xffffffffu, v1[i], 31);
+          a0[i] = (v0[i] << 1) | (p0 >> 31);
+          a1[i] = has1 ? ((v1[i] << 1) | (p1 >> 31)) : 0u;
+        }
+      }
+      uint32_t q0[KW], q1[KW];
 #pragma unroll
       for (int i = 0; i < KW; ++i) {
-        if (32 * i >= W) break;
         const int w = lane + 32 * i;
-        uint32_t p0 = __shfl_up_sync(0xffffffffu, v0[i], 1);
-        uint32_t p1 = __shfl_up_sync(0xffffffffu, v1[i], 1);
-        if (lane == 0) {
-          p0 = c0;
-          p1 = c1;
+        q0[i] = (w < W && a0[i]) ? d0[w] : 0u;
+        q1[i] = (w < W && a1[i]) ? d1[w] : 0u;
+      }
+      bool ch0 = false, ch1 = false;
+#pragma unroll
+      for (int i = 0; i < KW; ++i) {
+        const int w = lane + 32 * i;
+        if (w < W && (a0[i] & ~q0[i])) {
+          d0[w] = q0[i] | a0[i];
+          ch0 = true;
         }
-        c0 = __shfl_sync(0xffffffffu, v0[i], 31);
-        c1 = __shfl_sync(0xffffffffu, v1[i], 31);
-        const uint32_t a0 = (v0[i] << 1) | (p0 >> 31);
-        const uint32_t a1 = (v1[i] << 1) | (p1 >> 31);
-        if (w < W && a0) {
-          const uint32_t old = d0[w];
-          if ((old | a0) != old) {
-            d0[w] = old | a0;
-            ch0 = true;
-          }
-        }
-        if (w < W && a1 && has1) {
-          const uint32_t old = d1[w];
-          if ((old | a1) != old) {
-            d1[w] = old | a1;
-            ch1 = true;
-          }
+        if (w < W && (a1[i] & ~q1[i])) {
+          d1[w] = q1[i] | a1[i];
+          ch1 = true;
         }
       }
       ch0 = __any_sync(0xffffffffu, ch0);
@@ -461,8 +472,13 @@ class EarleyColsGS {
     if (REC && threadIdx.x == 0) rec->col_gap[c] = gap ? 1 : 0;
     const int mode = gap ? 1 : 0;  // the advance rule: next_any in a gap, nullable_next elsewhere
     // 1. origins below c, highest first; warp 0 walks down the dirty origins
-    //    until one completes something new, then every warp scatters
-    int top = c - 1;
+    //    until one completes something new, then every warp scatters.
+    //    A node (not a gap) reached only by epsilon edges from finished
+    //    columns needs none of it: each of its rows is a union of rows that
+    //    are closed under completion and advance, and so is the union (what
+    //    an origin completes here, it completed in one of the sources, whose
+    //    rows below already hold the advanced items).
+    int top = (!gap && !gs.labelled) ? -1 : c - 1;
     for (long long step = 0;; ++step) {
       if (warp == 0) {
         PH_BEGIN(t_or);
@@ -647,6 +663,7 @@ class EarleyColsGS {
       gs.vset[v] = 0;
       gs.vdone[v] = 0;
     }
+    if (threadIdx.x == 0) gs.labelled = 0;
     __syncthreads();
   }
 
@@ -655,7 +672,7 @@ class EarleyColsGS {
   // Warp: completed nonterminals and folded summaries of stored entry k.
   __device__ void record_entry(const uint32_t* row, long long k) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    uint32_t* nts = gs.wnt[warp];
+    uint32_t* nts = wnt + (size_t)warp * kMaxVW;
     for (int v = lane; v < VW; v += 32) nts[v] = 0;
     __syncwarp();
     uint32_t fnt = 0, ft = 0;
@@ -709,6 +726,7 @@ class EarleyColsGS {
       gs.vset[v] = 0;
       gs.vdone[v] = 0;
     }
+    if (threadIdx.x == 0) gs.labelled = 0;
     __syncthreads();
   }
 

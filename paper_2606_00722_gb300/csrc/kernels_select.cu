@@ -8,7 +8,9 @@ using namespace epic;
 
 // Alg. 4 per sequence: one CTA runs RelaxedSelect / ExactShrink with an
 // explicit stack; thread 0 drives the recursion, the whole CTA runs each
-// cover test (CoverCols walk) and exact joint check (EarleyCols walk).
+// cover test (CoverCols walk) and exact joint check (a walk with the
+// Gauss-Seidel columns of gscols.cuh, the grammar's per-item tables staged in
+// dynamic shared memory).
 
 struct SelFrame {
   int8_t kind;  // 0 root, 1 relaxed, 2 shrink
@@ -27,8 +29,12 @@ __global__ void __launch_bounds__(kThreads) k_select_spec(DevGrammar g, const Le
                                                           const int32_t* __restrict__ tok, int8_t* __restrict__ spec,
                                                           WsPack wsp) {
   __shared__ WalkShared sh;
+  __shared__ GsShared gss;
   __shared__ int s_pos[kMaxSel], s_tok[kMaxSel];
   __shared__ int ns;
+  extern __shared__ __align__(16) unsigned char dyn[];
+  GsTables tb;
+  gs_stage_tables(g, dyn, tb);
   Workspace ws;
   WalkScratch sc;
   wsp.carve(blockIdx.x, ws, sc);
@@ -51,8 +57,8 @@ __global__ void __launch_bounds__(kThreads) k_select_spec(DevGrammar g, const Le
     if (ns >= 2) {  // a set of at most one candidate is never tested
       Subst s{s_pos, s_tok, ns};
       if (exact) {
-        EarleyCols cols(g, table, ws, sc, wsp.dims, sh);
-        Walk<EarleyCols> w(cols, g, table, sc, sh, vocab);
+        EarleyColsGS<false> cols(g, tb, table, ws, sc, wsp.dims, sh, gss);
+        Walk<EarleyColsGS<false>> w(cols, g, table, sc, sh, vocab);
         r = w.run(x + (long long)b * n, n, s);
       } else {
         CoverCols cols(g, ws, wsp.dims, sh);
@@ -72,6 +78,10 @@ __global__ void __launch_bounds__(kThreads) k_select(DevGrammar g, const LexEntr
                                                      uint8_t* __restrict__ selected, WsPack wsp,
                                                      const int8_t* __restrict__ spec, unsigned long long* stats) {
   __shared__ WalkShared sh;
+  __shared__ GsShared gss;
+  extern __shared__ __align__(16) unsigned char dyn[];
+  GsTables tb;
+  gs_stage_tables(g, dyn, tb);
   __shared__ int c_slot[kMaxSel], c_pos[kMaxSel], c_tok[kMaxSel];
   __shared__ int s_pos[kMaxSel], s_tok[kMaxSel];
   __shared__ SelFrame stack[2 * kMaxSel + 8];
@@ -80,9 +90,9 @@ __global__ void __launch_bounds__(kThreads) k_select(DevGrammar g, const LexEntr
   Workspace ws;
   WalkScratch sc;
   wsp.carve(blockIdx.x, ws, sc);
-  EarleyCols ecols(g, table, ws, sc, wsp.dims, sh);
+  EarleyColsGS<false> ecols(g, tb, table, ws, sc, wsp.dims, sh, gss);
   CoverCols ccols(g, ws, wsp.dims, sh);
-  Walk<EarleyCols> exact(ecols, g, table, sc, sh, vocab);
+  Walk<EarleyColsGS<false>> exact(ecols, g, table, sc, sh, vocab);
   Walk<CoverCols> cover(ccols, g, table, sc, sh, vocab);
   for (int b = blockIdx.x; b < B; b += gridDim.x) {
     const int32_t* xb = x + (long long)b * n;
@@ -264,18 +274,180 @@ __global__ void __launch_bounds__(kThreads) k_select(DevGrammar g, const LexEntr
   }
 }
 
+// Alg. 1's sequential rejection fallback, one CTA per sequence: fill =
+// max(0, n_target[b] - |B|) more commits, each the highest-confidence
+// candidate (ties: position, then candidate index) at a still-masked
+// position that was not rejected and whose update passes the exact test
+// (a whole-graph walk of x (+) c with the Gauss-Seidel columns); a candidate
+// that fails is rejected for good (x only gains commits, and completability
+// is monotone).  Commits go straight into x.  Bounded by the k K candidates.
+__global__ void __launch_bounds__(kThreads) k_fallback(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
+                                                       int32_t* __restrict__ x, int B, int n,
+                                                       const int32_t* __restrict__ pos, int k,
+                                                       const int32_t* __restrict__ cand,
+                                                       const float* __restrict__ conf, int K,
+                                                       const int32_t* __restrict__ n_target,
+                                                       const uint8_t* __restrict__ selected,
+                                                       int32_t* __restrict__ filled, WsPack wsp,
+                                                       unsigned long long* stats) {
+  __shared__ WalkShared sh;
+  __shared__ GsShared gss;
+  extern __shared__ __align__(16) unsigned char dyn[];
+  GsTables tb;
+  gs_stage_tables(g, dyn, tb);
+  __shared__ uint8_t rej[kMaxFallbackCand];
+  __shared__ float r_cf[kThreads / 32];
+  __shared__ int r_q[kThreads / 32];
+  __shared__ int s_pos[1], s_tok[1];
+  __shared__ int s_fill, s_bad, s_q;
+  Workspace ws;
+  WalkScratch sc;
+  wsp.carve(blockIdx.x, ws, sc);
+  EarleyColsGS<false> cols(g, tb, table, ws, sc, wsp.dims, sh, gss);
+  Walk<EarleyColsGS<false>> walk(cols, g, table, sc, sh, vocab);
+  const int nc = k * K;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  unsigned long long n_chk = 0, n_com = 0, n_ovf = 0, n_bad = 0;
+  for (int b = blockIdx.x; b < B; b += gridDim.x) {
+    int32_t* xb = x + (long long)b * n;
+    for (int j = threadIdx.x; j < k; j += blockDim.x) filled[(long long)b * k + j] = -1;
+    for (int q = threadIdx.x; q < nc; q += blockDim.x) rej[q] = 0;
+    if (threadIdx.x == 0) {
+      int nsel = 0;
+      if (selected)
+        for (int j = 0; j < k; ++j) nsel += selected[(long long)b * k + j] == 1;
+      s_fill = n_target[b] - nsel;
+      s_bad = 0;
+      for (int q = 0; q < nc; ++q) {
+        const float cf = conf[(long long)b * nc + q];
+        if (cf != cf) s_bad = 1;
+        const int p = pos[(long long)b * k + q / K];
+        if (p < 0 || p >= n) s_bad = 1;
+      }
+    }
+    __syncthreads();
+    if (s_bad) {
+      if (threadIdx.x == 0) ++n_bad;
+      continue;
+    }
+    int done = 0;
+    for (int guard = 0; guard <= nc && done < s_fill; ++guard) {
+      // the next candidate: highest confidence, then lowest position, then
+      // lowest candidate index, among those not rejected at masked positions
+      float bc = 0.f;
+      int bq = -1;
+      for (int q = threadIdx.x; q < nc; q += blockDim.x) {
+        if (rej[q]) continue;
+        const int p = pos[(long long)b * k + q / K];
+        if (xb[p] >= 0) continue;  // committed by the selected batch or earlier here
+        const float cf = conf[(long long)b * nc + q];
+        const bool better = bq < 0 || cf > bc ||
+                            (cf == bc && (p < pos[(long long)b * k + bq / K] ||
+                                          (p == pos[(long long)b * k + bq / K] && q < bq)));
+        if (better) {
+          bc = cf;
+          bq = q;
+        }
+      }
+      for (int off = 16; off; off >>= 1) {
+        const float oc = __shfl_xor_sync(0xffffffffu, bc, off);
+        const int oq = __shfl_xor_sync(0xffffffffu, bq, off);
+        bool take = false;
+        if (oq >= 0) {
+          if (bq < 0 || oc > bc) {
+            take = true;
+          } else if (oc == bc) {
+            const int po = pos[(long long)b * k + oq / K], pb = pos[(long long)b * k + bq / K];
+            take = po < pb || (po == pb && oq < bq);
+          }
+        }
+        if (take) {
+          bc = oc;
+          bq = oq;
+        }
+      }
+      if (lane == 0) {
+        r_cf[warp] = bc;
+        r_q[warp] = bq;
+      }
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        float c0 = 0.f;
+        int q0 = -1;
+        for (int i = 0; i < (int)(blockDim.x >> 5); ++i) {
+          const int oq = r_q[i];
+          if (oq < 0) continue;
+          const float oc = r_cf[i];
+          bool take = q0 < 0 || oc > c0;
+          if (!take && oc == c0) {
+            const int po = pos[(long long)b * k + oq / K], pb = pos[(long long)b * k + q0 / K];
+            take = po < pb || (po == pb && oq < q0);
+          }
+          if (take) {
+            c0 = oc;
+            q0 = oq;
+          }
+        }
+        s_q = q0;
+        if (q0 >= 0) {
+          s_pos[0] = pos[(long long)b * k + q0 / K];
+          s_tok[0] = cand[(long long)b * nc + q0];
+        }
+      }
+      __syncthreads();
+      const int q = s_q;
+      if (q < 0) break;  // every candidate rejected
+      Subst su{s_pos, s_tok, 1};
+      const int r = walk.run(xb, n, su);
+      if (threadIdx.x == 0) {
+        ++n_chk;
+        if (r == 1) {
+          xb[s_pos[0]] = s_tok[0];
+          filled[(long long)b * k + q / K] = s_tok[0];
+          ++n_com;
+        } else {
+          rej[q] = 1;
+          if (r == -1) ++n_ovf;
+        }
+      }
+      __syncthreads();
+      if (r == 1) ++done;
+    }
+  }
+  if (threadIdx.x == 0) {
+    atomicAdd(&stats[S_FB_CHECKS], n_chk);
+    atomicAdd(&stats[S_FB_COMMITS], n_com);
+    atomicAdd(&stats[S_OVERFLOW], n_ovf);
+    atomicAdd(&stats[S_BAD], n_bad);
+  }
+}
+
 namespace epic {
 
 void launch_select_spec(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab,
                         const int32_t* x, int B, int n, const int32_t* pos, int k, const int32_t* tok, int8_t* spec,
                         const WsPack& wsp) {
-  k_select_spec<<<grid, kThreads, 0, st>>>(g, table, vocab, x, B, n, pos, k, tok, spec, wsp);
+  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps);
+  cudaFuncSetAttribute(k_select_spec, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+  k_select_spec<<<grid, kThreads, dyn, st>>>(g, table, vocab, x, B, n, pos, k, tok, spec, wsp);
 }
 
 void launch_select(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab,
                    const int32_t* x, int B, int n, const int32_t* pos, int k, const int32_t* tok, const float* conf,
                    uint8_t* selected, const WsPack& wsp, const int8_t* spec, unsigned long long* stats) {
-  k_select<<<grid, kThreads, 0, st>>>(g, table, vocab, x, B, n, pos, k, tok, conf, selected, wsp, spec, stats);
+  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps);
+  cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+  k_select<<<grid, kThreads, dyn, st>>>(g, table, vocab, x, B, n, pos, k, tok, conf, selected, wsp, spec, stats);
+}
+
+void launch_fallback(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab, int32_t* x,
+                     int B, int n, const int32_t* pos, int k, const int32_t* cand, const float* conf, int K,
+                     const int32_t* n_target, const uint8_t* selected, int32_t* filled, const WsPack& wsp,
+                     unsigned long long* stats) {
+  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps);
+  cudaFuncSetAttribute(k_fallback, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+  k_fallback<<<grid, kThreads, dyn, st>>>(g, table, vocab, x, B, n, pos, k, cand, conf, K, n_target, selected, filled,
+                                          wsp, stats);
 }
 
 }  // namespace epic

@@ -6,6 +6,7 @@
 #pragma once
 #include <cuda_runtime.h>
 
+#include "gscols.cuh"
 #include "packs.cuh"
 #include "seqpack.cuh"
 
@@ -43,11 +44,18 @@ void launch_select(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEnt
                    const int32_t* x, int B, int n, const int32_t* pos, int k, const int32_t* tok, const float* conf,
                    uint8_t* selected, const WsPack& wsp, const int8_t* spec, unsigned long long* stats);
 
+// Alg. 1's sequential rejection fallback
+void launch_fallback(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab, int32_t* x,
+                     int B, int n, const int32_t* pos, int k, const int32_t* cand, const float* conf, int K,
+                     const int32_t* n_target, const uint8_t* selected, int32_t* filled, const WsPack& wsp,
+                     unsigned long long* stats);
+
 // measurement builds (EPIC_PHASE_TIMERS): the walk's phase counters of one
 // translation unit, added into out16 (reset: zeroed afterwards)
 int phase_read_walk(unsigned long long* out16, int reset);
 int phase_read_forward(unsigned long long* out16, int reset);
 int phase_read_check_sm(unsigned long long* out16, int reset);
 int phase_read_check_global(unsigned long long* out16, int reset);
+int phase_read_good(unsigned long long* out16, int reset);
 
 }  // namespace epic

@@ -50,7 +50,11 @@ inline size_t ws_bytes_per_cta(const WsDims& d, int W, int VW, int FW) {
          r((size_t)d.emax * W * 4);
 }
 
-enum StatIdx { S_CHECKS, S_VALID, S_OVERFLOW, S_BAD, S_COLUMNS, S_ENTRIES, S_COVER, S_EXACT, S_SELECTED, S_N };
+enum StatIdx {
+  S_CHECKS, S_VALID, S_OVERFLOW, S_BAD, S_COLUMNS, S_ENTRIES, S_COVER, S_EXACT, S_SELECTED,
+  S_FB_CHECKS, S_FB_COMMITS, S_N
+};
+constexpr int kMaxFallbackCand = 4096;  // proposed (position, candidate) pairs per sequence of the fallback
 
 // shared-memory staging of one warp: rows, completed-NT sets, slot origins,
 // origin slots (16-byte multiple)

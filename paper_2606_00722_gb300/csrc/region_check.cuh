@@ -156,6 +156,7 @@ struct RegionCheck {
         if (!fold) continue;
         expn_of_set(w.g, w.sh.nt, w.sh.expn);
         __syncwarp();
+        w.col_labelled = true;  // new items to close, not a copy of a closed column
         w.scatter(u, w.sh.expn, true, 0, fold);
         if (w.status) return -1;
       }

@@ -112,6 +112,7 @@ __global__ void __launch_bounds__(32 * kGsMaxWarps, 1) k_forward_gs(DevGrammar g
     d.emax = sp.emax;
     EarleyColsGS<true> cols(g, tb, table, ws, sc, d, sh, gss);
     cols.rec = &br;
+    cols.wnt = (uint32_t*)(dyn + gs_tables_bytes(g.D, g.W, g.adv_steps));
     Walk<EarleyColsGS<true>> walk(cols, g, table, sc, sh, vocab);
     walk.rec = &br;
     Subst none{nullptr, nullptr, 0};
@@ -145,7 +146,7 @@ void launch_forward(bool sm, dim3 grid, dim3 block, size_t dyn, cudaStream_t st,
 
 void launch_forward_gs(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab,
                        const int32_t* x, int B, int n, const SeqPack& sp, unsigned long long* stats) {
-  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps);
+  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps) + (size_t)kGsMaxWarps * kMaxVW * 4;
   cudaFuncSetAttribute(k_forward_gs, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
   k_forward_gs<<<grid, 32 * kGsMaxWarps, dyn, st>>>(g, table, vocab, x, B, n, sp, stats);
 }

@@ -68,8 +68,10 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
   __shared__ int s_self;
   __shared__ uint32_t s_cn[kWMaxVW], s_bset[kWMaxVW];
   __shared__ uint32_t s_expn[kWMaxW];
+  __shared__ uint32_t s_xall[kWMaxW];
   __shared__ int s_flag;
   for (long long b = blockIdx.x; b < B; b += gridDim.x) {
+  PH_BEGIN(t_setup);
   SeqArena a = sp.carve(b);
   int32_t* meta = a.rec.meta;
   if (meta[M_STATUS] != 1) continue;
@@ -119,6 +121,7 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
     for (long long k = col[j] + lane; k < col[j + 1]; k += 32) a.succ_idx[atomicAdd(&cur_s[org[k]], 1)] = j;
   __syncthreads();
 
+  PH_END(0, t_setup);
   uint32_t* G = a.good;
   uint32_t* sfold = (uint32_t*)a.cursor;  // per successor of the column (the cursors are free now)
   for (int j = N - 1; j >= 0; --j) {
@@ -127,6 +130,7 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
     const long long k0 = col[j], k1 = col[j + 1];
     if (k0 == k1) continue;
     // EXPN of what completes from origin j at each column j2 (j2 = j included)
+    PH_BEGIN(t_succ);
     if (tid == 0) s_self = -1;
     __syncthreads();
     for (int si = s0 + tid; si < s1; si += nthr)
@@ -142,7 +146,17 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
       if (lane == 0) sfold[si - s0] = f;  // folded (bit C mod 32): 0 = nothing completes
     }
     __syncthreads();
+    // union of the completion masks of the successors after j
+    for (int w = tid; w < W; w += nthr) {
+      uint32_t u = 0;
+      for (int si = s0; si < s1; ++si)
+        if (si - s0 != self_si && sfold[si - s0]) u |= a.expn[(size_t)(si - s0) * W + w];
+      s_xall[w] = u;
+    }
+    __syncthreads();
+    PH_END(1, t_succ);
     // in-row rules of this column: the gap self-loop and nullable completions
+    PH_BEGIN(t_a);
     uint32_t inrow[KW];
 #pragma unroll
     for (int i = 0; i < KW; ++i) {
@@ -203,7 +217,19 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
         }
       }
       const uint32_t wfold = a.ws.esum[(size_t)k * 2];  // waited nonterminals, folded
+      // the most the nested rule can make good: items waiting on a
+      // nonterminal that completes from j somewhere after j
+      uint32_t want[KW];
+#pragma unroll
+      for (int i = 0; i < KW; ++i) {
+        const int w = lane + 32 * i;
+        want[i] = (w < W) ? (bits[i] & s_xall[w]) : 0u;
+      }
       for (int sb = s0; sb < s1; sb += 32) {
+        bool open = false;
+#pragma unroll
+        for (int i = 0; i < KW; ++i) open |= (want[i] & ~acc[i]) != 0;
+        if (!__any_sync(0xffffffffu, open)) break;
         const int si = sb + lane;
         int k3 = -1;
         if (si < s1 && si - s0 != self_si && (sfold[si - s0] & wfold) != 0) {
@@ -242,6 +268,7 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
       if (lane == 0) a.gnz[k] = nz ? 1 : 0;
     }
     __syncthreads();
+    PH_END(2, t_a);
     // B. completions within the column, entries with complete items in
     //    ascending origin order
     for (long long k = k0; k < k1; ++k) {
@@ -270,27 +297,50 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
         s_expn[w] = acc;
       }
       __syncthreads();
-      // which of them some entry (o, o2 < o) of column o turns good at (j, o2)
+      PH_BEGIN(t_g);
+      // which of them some entry (o, o2 < o) of column o turns good at (j, o2):
+      // one warp per entry of column o, lanes over words; the gather stops
+      // once every completed nonterminal is found
       const int cb = col[o], ce = col[o + 1];
       const bool self = ce > cb && org[ce - 1] == o;
       const int nent = self ? ce - cb - 1 : ce - cb;
-      const long long total = (long long)nent * W;
-      for (long long t = tid; t < total; t += nthr) {
-        const int kp = cb + (int)(t / W), w = (int)(t % W);
-        const int kk = a.eidx[tri_index(j, org[kp])];
-        if (kk < 0 || !a.gnz[kk]) continue;
-        uint32_t m = a.ws.bits[(size_t)kp * W + w] & s_expn[w] & shr1_word(G + (size_t)kk * W, w, W);
-        while (m) {
-          const int bb = __ffs(m) - 1;
-          m &= m - 1;
-          const int Bn = tb.item_next[(w << 5) + bb] - g.T;
-          const uint32_t bit = 1u << (Bn & 31);
-          if (!(s_bset[Bn >> 5] & bit)) atomicOr(&s_bset[Bn >> 5], bit);
+      for (int e0 = 0; e0 < nent; e0 += kGoodWarps) {
+        const int e = e0 + warp;
+        if (e < nent) {
+          const int kp = cb + e;
+          const int kk = a.eidx[tri_index(j, org[kp])];
+          if (kk >= 0 && a.gnz[kk]) {
+            const uint32_t* P = a.ws.bits + (size_t)kp * W;
+            const uint32_t* GK = G + (size_t)kk * W;
+            for (int w = lane; w < W; w += 32) {
+              const uint32_t xw = s_expn[w];
+              if (!xw) continue;
+              uint32_t m = P[w] & xw;
+              if (m) m &= shr1_word(GK, w, W);
+              while (m) {
+                const int bb = __ffs(m) - 1;
+                m &= m - 1;
+                const int Bn = tb.item_next[(w << 5) + bb] - g.T;
+                const uint32_t bit = 1u << (Bn & 31);
+                if (!(s_bset[Bn >> 5] & bit)) atomicOr(&s_bset[Bn >> 5], bit);
+              }
+            }
+          }
         }
+        __syncthreads();
+        if (tid == 0) {
+          uint32_t left = 0;
+          for (int v = 0; v < VW; ++v) left |= s_cn[v] & ~s_bset[v];
+          s_flag = left != 0;
+        }
+        __syncthreads();
+        if (!s_flag) break;
       }
       __syncthreads();
+      PH_END(3, t_g);
       // one warp: complete items with a good left side, the in-row closure,
       // and the self-loop through the entry of column o with origin o
+      PH_BEGIN(t_w);
       if (warp == 0) {
         const uint32_t* bp = a.ws.bits + (size_t)k * W;
         const uint32_t* E = self ? a.ws.bits + (size_t)(ce - 1) * W : nullptr;
@@ -359,6 +409,7 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
         }
       }
       __syncthreads();
+      PH_END(4, t_w);
     }
   }
   __syncthreads();
@@ -373,5 +424,22 @@ void launch_good(dim3 grid, cudaStream_t st, const DevGrammar& g, int B, const S
 }
 
 int good_warps() { return kGoodWarps; }
+
+// measurement builds: this translation unit's phase counters
+int phase_read_good(unsigned long long* out16, int reset) {
+#ifdef EPIC_PHASE_TIMERS
+  unsigned long long h[16];
+  if (cudaMemcpyFromSymbol(h, g_phase, sizeof(h)) != cudaSuccess) return -1;
+  for (int i = 0; i < 16; ++i) out16[i] += h[i];
+  if (reset) {
+    unsigned long long z[16] = {0};
+    if (cudaMemcpyToSymbol(g_phase, z, sizeof(z)) != cudaSuccess) return -1;
+  }
+#else
+  (void)out16;
+  (void)reset;
+#endif
+  return 0;
+}
 
 }  // namespace epic

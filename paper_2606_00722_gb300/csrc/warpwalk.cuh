@@ -168,6 +168,7 @@ class WarpWalker {
   SeqRec* rec = nullptr;
   int cur_col = -1;
   uint32_t cur_lbl8[8];      // label set of the arrivals being made (all zero = epsilon)
+  bool col_labelled = false; // the open column has a labelled arrival (else only epsilon ones)
 
   __device__ WarpWalker(const DevGrammar& g_, const LexEntry* t, WWs w, WSh& s, int nm, long long em, int voc)
       : g(g_), table(t), ws(w), sh(s), nmax(nm), emax(em), vocab(voc), W(g_.W), VW(g_.VW) {}
@@ -605,6 +606,7 @@ class WarpWalker {
     rec->n_edges = __shfl_sync(0xffffffffu, rec->n_edges, 0);
   }
   __device__ void arrive_inner(int src, const uint32_t* M, bool shift) {
+    col_labelled |= shift;
     if constexpr (EXT)
       if (rec) record_edge(src, shift);
     if (shift)
@@ -640,6 +642,11 @@ class WarpWalker {
   __device__ void close_column(int c, bool gap) {
     cur_gap = gap;
     const uint32_t* P = gap ? g.gap_pred : g.pred;
+    // A node (not a gap) reached only by epsilon edges from finished columns:
+    // each row below c is a union of rows closed under completion and
+    // advance, and so is the union, so those rows only contribute their
+    // waited nonterminals (the predictions at c).
+    const bool eps_only = !gap && !col_labelled;
     for (long long it = 0;; ++it) {
       if (it > kWMaxSteps) {
         status = 1;
@@ -683,6 +690,10 @@ class WarpWalker {
       if (wl_lane() == 0) sh.dirty[o >> 5] &= ~(1u << (o & 31));
       __syncwarp();
       uint32_t* row = row_of(o);
+      if (eps_only && o < c) {
+        row_scan(row, sh.vset, sum_of(o));
+        continue;
+      }
       if (o == c) {  // completions from c at c: the nullable / gap advance rules
         PH_BEGIN(t_row);
         row_advance(row, gap ? g.next_any : g.nullable_next);
@@ -802,11 +813,13 @@ class WarpWalker {
     __syncwarp();
     nent = E;
     ncols = c + 1;
+    col_labelled = false;
   }
   __device__ bool column_empty(int c) { return cend(c) == cbeg(c); }
 
   // abandon the open column: zero its rows
   __device__ void cleanup() {
+    col_labelled = false;
     int o = -1;
     while ((o = bm_next(sh.touched, o + 1, kWCols)) >= 0) {
       if constexpr (!SM) {

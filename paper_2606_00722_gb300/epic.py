@@ -72,7 +72,8 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
 class _Stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in ('checks', 'valid', 'overflow', 'bad_inputs', 'columns',
                                           'entries', 'cover_checks', 'exact_checks', 'selected',
-                                          'region_checks', 'validate_kernels')]
+                                          'region_checks', 'validate_kernels', 'fallback_checks',
+                                          'fallback_commits')]
 
 
 class _Desc(C.Structure):
@@ -86,7 +87,7 @@ _lib = None
 EXPORTS = ('epic_grammar_create', 'epic_grammar_destroy', 'epic_grammar_lexer_states',
            'epic_lexer_table_build', 'epic_lexer_table_destroy', 'epic_lexer_table_copy',
            'epic_validate_batch', 'epic_validate_batch_noalloc',
-           'epic_pick_candidates', 'epic_select_compatible_subset', 'epic_commit',
+           'epic_pick_candidates', 'epic_select_compatible_subset', 'epic_commit', 'epic_fallback_commit',
            'epic_get_stats', 'epic_status_string', 'epic_measure_int_peak', 'epic_last_kernel_times')
 
 
@@ -111,6 +112,7 @@ def load(path: str | None = None):
     lib.epic_pick_candidates.argtypes = [vp, vp, vp, i32, i32, i32, vp, vp, vp]
     lib.epic_select_compatible_subset.argtypes = [vp, vp, vp, i32, i32, vp, i32, vp, vp, vp, vp]
     lib.epic_commit.argtypes = [vp, i32, i32, vp, i32, vp, vp, vp]
+    lib.epic_fallback_commit.argtypes = [vp, vp, vp, i32, i32, vp, i32, vp, vp, i32, vp, vp, vp, vp]
     lib.epic_get_stats.argtypes = [vp, C.POINTER(_Stats), C.c_size_t, C.c_int]
     lib.epic_measure_int_peak.argtypes = [C.POINTER(C.c_double), C.POINTER(C.c_double), vp]
     lib.epic_measure_int_peak.restype = C.c_int
@@ -224,10 +226,11 @@ class LexTable:
 
     def kernel_times(self) -> dict:
         """epic_last_kernel_times: {kernel name: ms} of the last
-        validate_batch call on this table (synchronizes)."""
-        ms = (C.c_float * 4)()
-        names = (C.c_char_p * 4)()
-        n = load().epic_last_kernel_times(self.h, ms, names, 4)
+        validate_batch and select_compatible_subset calls on this table
+        (synchronizes)."""
+        ms = (C.c_float * 8)()
+        names = (C.c_char_p * 8)()
+        n = load().epic_last_kernel_times(self.h, ms, names, 8)
         if n < 0:
             raise EpicError(ERR_CUDA, 'epic_last_kernel_times')
         return {names[i].decode(): float(ms[i]) for i in range(n)}
@@ -294,3 +297,28 @@ def commit(x, pos, tok, selected, stream=None):
     k = pos.shape[1]
     _check(load().epic_commit(_ptr(x), B, n, _ptr(pos), k, _ptr(tok), _ptr(selected), _stream(stream)),
            'epic_commit')
+
+
+def fallback_commit(g: Grammar, t: LexTable, x, pos, cand, cand_conf, n_target, selected, filled, stream=None):
+    """epic_fallback_commit: Alg. 1's sequential rejection fallback (selected
+    may be None for an empty batch B)."""
+    B, n = x.shape
+    k = pos.shape[1]
+    K = cand.shape[2]
+    _check(load().epic_fallback_commit(g.h, t.h, _ptr(x), B, n, _ptr(pos), k, _ptr(cand), _ptr(cand_conf), K,
+                                       _ptr(n_target), _ptr(selected), _ptr(filled), _stream(stream)),
+           'epic_fallback_commit')
+
+
+def decode_step(g: Grammar, t: LexTable, x, pos, cand, cand_conf, n_target, bufs, stream=None):
+    """One denoising step's constraint work (Alg. 1 after the model's
+    proposal): validate every (position, candidate), pick C, select and commit
+    the relaxed-compatible batch B (Alg. 4), then fill the commits still
+    wanted by the rejection fallback.  bufs holds the device outputs: valid
+    [B][k][K] uint8, tok [B][k] int32, conf [B][k] float32, selected [B][k]
+    uint8, filled [B][k] int32.  Only sequences the C-ABI calls; asynchronous."""
+    validate_batch(g, t, x, pos, cand, bufs['valid'], stream)
+    pick_candidates(cand, cand_conf, bufs['valid'], bufs['tok'], bufs['conf'], stream)
+    select_compatible_subset(g, t, x, pos, bufs['tok'], bufs['conf'], bufs['selected'], stream)
+    commit(x, pos, bufs['tok'], bufs['selected'], stream)
+    fallback_commit(g, t, x, pos, cand, cand_conf, n_target, bufs['selected'], bufs['filled'], stream)

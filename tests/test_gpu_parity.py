@@ -108,3 +108,41 @@ def test_pick_golden(cuda, shape):
     torch.cuda.synchronize()
     np.testing.assert_array_equal(tok.cpu().numpy().reshape(-1), etok)
     np.testing.assert_array_equal(cf.cpu().numpy().reshape(-1).view(np.uint32), econf.view(np.uint32))
+
+
+@pytest.mark.parametrize('name,seed,kw,fill', [
+    ('expr-tiny', 42, {}, 8), ('expr-tiny', 45, dict(k=6, K=4), 6),
+    ('json-schema', 43, dict(batch=3, k=6, K=6), 6), ('smiles-256', 44, dict(batch=3, k=6, K=5), 4),
+    ('clike-512', 42, dict(batch=1, k=2, K=4, n=128), 2),
+])
+def test_decode_step_with_fallback(cuda, name, seed, kw, fill):
+    """One whole step (validate, pick, select, commit, then Alg. 1's rejection
+    fallback for the commits still wanted) against the oracle's, bit-exact:
+    validity bits, selected batch, fallback commits and the final x."""
+    import torch
+    import paper_2606_00722_gb300 as epic
+    w = make_workload(name, seed, **kw)
+    O = oracle.Oracle(w.grammar, w.vocab)
+    n_target = np.full(w.B, fill, np.int32)
+    g = epic.Grammar(w.grammar)
+    t = epic.LexTable(g, w.vocab)
+    x = _dev(w.x, cuda)
+    bufs = dict(valid=torch.empty(w.cand.shape, dtype=torch.uint8, device=cuda),
+                tok=torch.empty(w.pos.shape, dtype=torch.int32, device=cuda),
+                conf=torch.empty(w.pos.shape, dtype=torch.float32, device=cuda),
+                selected=torch.empty(w.pos.shape, dtype=torch.uint8, device=cuda),
+                filled=torch.empty(w.pos.shape, dtype=torch.int32, device=cuda))
+    epic.decode_step(g, t, x, _dev(w.pos, cuda), _dev(w.cand, cuda), _dev(w.conf, cuda), _dev(n_target, cuda), bufs)
+    torch.cuda.synchronize()
+    st = t.stats()
+    ref_valid = O.validate_batch(w.x, w.pos, w.cand, nthreads=NTHREADS)
+    rtok, rconf = oracle.pick_candidates(ref_valid, w.cand, w.conf)
+    ref_sel = O.select(w.x, w.pos, rtok, rconf)
+    x1 = O.commit(w.x, w.pos, rtok, ref_sel)
+    ref_x, ref_filled, nchk = O.fallback(x1, w.pos, w.cand, w.conf, n_target, ref_sel)
+    np.testing.assert_array_equal(bufs['valid'].cpu().numpy(), ref_valid)
+    np.testing.assert_array_equal(bufs['selected'].cpu().numpy(), ref_sel)
+    np.testing.assert_array_equal(bufs['filled'].cpu().numpy(), ref_filled)
+    np.testing.assert_array_equal(x.cpu().numpy(), ref_x)
+    assert st['fallback_checks'] == nchk
+    assert st['fallback_commits'] == int((ref_filled >= 0).sum())
