@@ -1,9 +1,11 @@
 """Benchmark of one denoising step's constraint work on GB300.
 
 A step = epic_validate_batch + epic_pick_candidates +
-epic_select_compatible_subset + epic_commit over one batch of the workload
-(every proposed (position, candidate) pair checked, the compatible subset
-selected and committed).  Prints one JSON line.
+epic_select_compatible_subset + epic_commit + epic_fallback_commit over one
+batch of the workload: every proposed (position, candidate) pair checked, the
+relaxed-compatible subset selected, checked jointly and committed, then Alg.
+1's rejection fallback fills the commits still wanted (n_t = k per sequence).
+Prints one JSON line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   (the CPU oracle on the same config)
@@ -40,12 +42,13 @@ def parse():
     ap.add_argument('--gpus', type=int, default=1)
     ap.add_argument('--steps', type=int, default=5)
     ap.add_argument('--warmup', type=int, default=3)
-    ap.add_argument('--workload', default='json-schema')
+    ap.add_argument('--workload', default='clike-512')
     ap.add_argument('--impl', default='epic', choices=['epic', 'reference'])
     ap.add_argument('--seed', type=int, default=42)
     ap.add_argument('--cpu-seconds', type=float, default=15.0)
     ap.add_argument('--no-cpu-baseline', action='store_true')
     ap.add_argument('--k', type=int, default=None, help='proposed positions per sequence (sweep)')
+    ap.add_argument('--batch', type=int, default=None, help='sequences per batch (smaller cases for profiling)')
     return ap.parse_args()
 
 
@@ -181,14 +184,16 @@ def cpu_baseline(w, seconds):
     if w.n >= 1024:
         return cpu_baseline_bounded(w, seconds, cores)
     O = oracle.Oracle(w.grammar, w.vocab)
-    per_seq = w.k * w.K
+    # proposed positions in batch order, all K candidates of one per call (on
+    # every core), until the budget is spent
     t0 = time.perf_counter()
     done = 0
-    b = 0
-    while b < w.B and (time.perf_counter() - t0) < seconds:
-        O.validate_batch(w.x[b:b + 1], w.pos[b:b + 1], w.cand[b:b + 1], nthreads=cores)
-        done += per_seq
-        b += 1
+    calls = 0
+    while calls < w.B * w.k and (time.perf_counter() - t0) < seconds:
+        b, j = divmod(calls, w.k)
+        O.validate_batch(w.x[b:b + 1], w.pos[b:b + 1, j:j + 1], w.cand[b:b + 1, j:j + 1], nthreads=cores)
+        done += w.K
+        calls += 1
     dt = time.perf_counter() - t0
     # the same oracle on one core: the first sequence's positions in turn (all
     # their candidates per call), for at most a fifth of the budget
@@ -201,8 +206,8 @@ def cpu_baseline(w, seconds):
         one += w.K
     dt1 = time.perf_counter() - t1
     return {'value': done / dt, 'unit': 'checks/s', 'cores': cores, 'kind': 'oracle',
-            'sample': '%d of %d sequences (%d checks), oracle validate_batch on %d threads, %.1f s'
-                      % (b, w.B, done, cores, dt),
+            'sample': '%d of %d proposed positions in batch order (%d checks), oracle validate_batch on %d '
+                      'threads, %.1f s' % (calls, w.B * w.k, done, cores, dt),
             'value_1core': one / dt1,
             'sample_1core': '%d checks of the first sequence, one position per call on 1 thread, %.1f s'
                             % (one, dt1)}
@@ -254,7 +259,7 @@ def run_reference(args):
     if rank != 0:
         return
     from synth import make_workload
-    w = make_workload(args.workload, args.seed, k=args.k)
+    w = make_workload(args.workload, args.seed, k=args.k, batch=args.batch)
     import oracle
     O = oracle.Oracle(w.grammar, w.vocab)
     cores = os.cpu_count() or 1
@@ -297,7 +302,7 @@ def main():
     import paper_2606_00722_gb300 as epic
     epic.build()
     from synth import make_workload
-    w = make_workload(args.workload, args.seed + rank, k=args.k)
+    w = make_workload(args.workload, args.seed + rank, k=args.k, batch=args.batch)
     g = epic.Grammar(w.grammar)
     t = epic.LexTable(g, w.vocab)
     x0 = torch.from_numpy(w.x).to(dev)
@@ -309,6 +314,8 @@ def main():
     tok = torch.empty(w.pos.shape, dtype=torch.int32, device=dev)
     conf = torch.empty(w.pos.shape, dtype=torch.float32, device=dev)
     sel = torch.empty(w.pos.shape, dtype=torch.uint8, device=dev)
+    filled = torch.empty(w.pos.shape, dtype=torch.int32, device=dev)
+    n_target = torch.full((w.B,), w.k, dtype=torch.int32, device=dev)  # n_t: commit every proposed position
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)  # > 129 MB L2
     stream = torch.cuda.current_stream()
     checks = w.B * w.k * w.K
@@ -318,6 +325,7 @@ def main():
         epic.pick_candidates(cand, conf3, valid, tok, conf)
         epic.select_compatible_subset(g, t, xbuf, pos, tok, conf, sel)
         epic.commit(xbuf, pos, tok, sel)
+        epic.fallback_commit(g, t, xbuf, pos, cand, conf3, n_target, sel, filled)
 
     for _ in range(args.warmup):
         x.copy_(x0)
@@ -341,6 +349,7 @@ def main():
             epic.pick_candidates(cand, conf3, valid, tok, conf)
             epic.select_compatible_subset(g, t, x, pos, tok, conf, sel)
             epic.commit(x, pos, tok, sel)
+            epic.fallback_commit(g, t, x, pos, cand, conf3, n_target, sel, filled)
             ev[i][2].record(stream)
             for kname, kms in t.kernel_times().items():  # waits for this step's kernels
                 kern.setdefault(kname, []).append(kms)
@@ -354,7 +363,12 @@ def main():
     # kernels of the timed region: validate's own (one walk kernel, or the
     # forward chart, good masks and region checks) + pick + two selection
     # kernels + commit
-    launches = st['validate_kernels'] + 4 * args.steps  # + pick, select_spec, select, commit
+    launches = st['validate_kernels'] + 5 * args.steps  # + pick, select_spec, select, commit, fallback
+    sel_h = sel.cpu().numpy()
+    fill_h = filled.cpu().numpy()
+    commit_sizes = {'selected_per_seq': float((sel_h == 1).sum()) / w.B,
+                    'fallback_per_seq': float((fill_h >= 0).sum()) / w.B,
+                    'selection_overflow': int((sel_h == 2).sum())}
     ms = float(np.mean(step_ms))
     vms = float(np.mean(val_ms))
     if world > 1:
@@ -369,8 +383,10 @@ def main():
     hvalid = torch.empty(w.cand.shape, dtype=torch.uint8).pin_memory()
     hsel = torch.empty(w.pos.shape, dtype=torch.uint8).pin_memory()
     hxo = torch.empty(w.x.shape, dtype=torch.int32).pin_memory()
+    hnt = torch.full((w.B,), w.k, dtype=torch.int32).pin_memory()
+    hfill = torch.empty(w.pos.shape, dtype=torch.int32).pin_memory()
     e2e_ms = []
-    for i in range(args.steps):
+    for i in range(min(args.steps, 3)):  # the same steps end to end (at most three: long steps)
         flush.fill_(i & 255)
         a, c = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
@@ -378,16 +394,18 @@ def main():
         pos.copy_(hpos, non_blocking=True)
         cand.copy_(hcand, non_blocking=True)
         conf3.copy_(hconf, non_blocking=True)
+        n_target.copy_(hnt, non_blocking=True)
         step(x)
         hvalid.copy_(valid, non_blocking=True)
         hsel.copy_(sel, non_blocking=True)
+        hfill.copy_(filled, non_blocking=True)
         hxo.copy_(x, non_blocking=True)
         c.record(stream)
         torch.cuda.synchronize()
         e2e_ms.append(a.elapsed_time(c))
     e2e_step = float(np.mean(e2e_ms))
-    h2d = w.x.nbytes + w.pos.nbytes + w.cand.nbytes + w.conf.nbytes
-    d2h = w.cand.size + w.pos.size + w.x.nbytes
+    h2d = w.x.nbytes + w.pos.nbytes + w.cand.nbytes + w.conf.nbytes + hnt.numel() * 4
+    d2h = w.cand.size + w.pos.size + w.pos.size * 4 + w.x.nbytes
     # ---- roofline of the dominant kernel of epic_validate_batch: bit-parallel
     # Earley word operations, 3 passes (predict, scan, complete) over every
     # (node, origin) pair of the chart the kernel builds, ceil(D / 32) words
@@ -428,6 +446,7 @@ def main():
             'step_latency_us': ms * 1e3, 'validate_checks_per_s': total_checks / (vms / 1e3),
             'valid_fraction': st['valid'] / max(1, st['checks']), 'overflow': st['overflow'],
             'gpu_launches': int(launches), 'validate_path': 'region' if region else 'walk',
+            'commits': commit_sizes,
             'e2e': {'value': total_checks / (e2e_step / 1e3), 'unit': 'checks/s', 'h2d_bytes_per_step': int(h2d),
                     'd2h_bytes_per_step': int(d2h)},
             'roofline': roof, 'clocks': clk.summary()}

@@ -89,9 +89,18 @@ struct RegionCheck {
     w.frontier_from(src, at_begin);
     for (int p = left_lo; p < left_hi && w.nf > 0; ++p)
       if (!w.span_step(x[p])) return -1;
-    if (w.nf > 0 && !w.span_step(t)) return -1;
-    for (int p = right_lo; p < right_hi && w.nf > 0; ++p)
-      if (!w.span_step(x[p])) return -1;
+    // the region's last span step feeds the gap after it (unless the region
+    // runs to the end): its end nodes reached by epsilon need no closure
+    w.defer_to_gap = !to_end && right_hi == right_lo;
+    const bool ok_t = w.nf == 0 || w.span_step(t);
+    w.defer_to_gap = false;
+    if (!ok_t) return -1;
+    for (int p = right_lo; p < right_hi && w.nf > 0; ++p) {
+      w.defer_to_gap = !to_end && p + 1 == right_hi;
+      const bool ok = w.span_step(x[p]);
+      w.defer_to_gap = false;
+      if (!ok) return -1;
+    }
     if (w.nf == 0) return 0;
     if (to_end) {
       int c = w.end_from_frontier();

@@ -69,6 +69,7 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
   __shared__ uint32_t s_cn[kWMaxVW], s_bset[kWMaxVW];
   __shared__ uint32_t s_expn[kWMaxW];
   __shared__ uint32_t s_xall[kWMaxW];
+  __shared__ uint32_t s_items[kWMaxW];  // good-advanceable waiting items of the gather
   __shared__ int s_flag;
   for (long long b = blockIdx.x; b < B; b += gridDim.x) {
   PH_BEGIN(t_setup);
@@ -124,6 +125,8 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
   PH_END(0, t_setup);
   uint32_t* G = a.good;
   uint32_t* sfold = (uint32_t*)a.cursor;  // per successor of the column (the cursors are free now)
+  for (int w = tid; w < kWMaxW; w += nthr) s_items[w] = 0;
+  __syncthreads();
   for (int j = N - 1; j >= 0; --j) {
     const int s0 = a.succ_off[j], s1 = a.succ_off[j + 1];
     const bool gap = a.rec.col_gap[j] != 0;
@@ -299,42 +302,60 @@ __global__ void __launch_bounds__(32 * kGoodWarps, 1) k_good(DevGrammar g, int B
       __syncthreads();
       PH_BEGIN(t_g);
       // which of them some entry (o, o2 < o) of column o turns good at (j, o2):
-      // one warp per entry of column o, lanes over words; the gather stops
-      // once every completed nonterminal is found
+      // each warp ORs, over its entries of column o, the waiting items whose
+      // advance is good into registers (one operation per word); the items
+      // become nonterminals once, at the end
       const int cb = col[o], ce = col[o + 1];
       const bool self = ce > cb && org[ce - 1] == o;
       const int nent = self ? ce - cb - 1 : ce - cb;
-      for (int e0 = 0; e0 < nent; e0 += kGoodWarps) {
-        const int e = e0 + warp;
-        if (e < nent) {
+      {
+        uint32_t ex[KW], acc[KW];
+#pragma unroll
+        for (int i = 0; i < KW; ++i) {
+          const int w = lane + 32 * i;
+          ex[i] = (w < W) ? s_expn[w] : 0u;
+          acc[i] = 0u;
+        }
+        for (int e = warp; e < nent; e += kGoodWarps) {
           const int kp = cb + e;
           const int kk = a.eidx[tri_index(j, org[kp])];
-          if (kk >= 0 && a.gnz[kk]) {
-            const uint32_t* P = a.ws.bits + (size_t)kp * W;
-            const uint32_t* GK = G + (size_t)kk * W;
-            for (int w = lane; w < W; w += 32) {
-              const uint32_t xw = s_expn[w];
-              if (!xw) continue;
-              uint32_t m = P[w] & xw;
-              if (m) m &= shr1_word(GK, w, W);
-              while (m) {
-                const int bb = __ffs(m) - 1;
-                m &= m - 1;
-                const int Bn = tb.item_next[(w << 5) + bb] - g.T;
-                const uint32_t bit = 1u << (Bn & 31);
-                if (!(s_bset[Bn >> 5] & bit)) atomicOr(&s_bset[Bn >> 5], bit);
-              }
-            }
+          if (kk < 0 || !a.gnz[kk]) continue;
+          const uint32_t* P = a.ws.bits + (size_t)kp * W;
+          const uint32_t* GK = G + (size_t)kk * W;
+          uint32_t pv[KW], gv[KW];
+#pragma unroll
+          for (int i = 0; i < KW; ++i) {
+            const int w = lane + 32 * i;
+            pv[i] = ex[i] ? (P[w] & ex[i]) : 0u;
+            gv[i] = (w < W) ? GK[w] : 0u;
+          }
+#pragma unroll
+          for (int i = 0; i < KW; ++i) {
+            if (32 * i >= W) break;
+            // bit b of word w takes bit b + 1 of G (bit 0 of word w + 1 for b = 31)
+            uint32_t nxt = __shfl_down_sync(0xffffffffu, gv[i], 1);
+            const uint32_t wrap = (i + 1 < KW) ? __shfl_sync(0xffffffffu, gv[i + 1], 0) : 0u;
+            if (lane == 31) nxt = wrap;
+            acc[i] |= pv[i] & ((gv[i] >> 1) | (nxt << 31));
           }
         }
-        __syncthreads();
-        if (tid == 0) {
-          uint32_t left = 0;
-          for (int v = 0; v < VW; ++v) left |= s_cn[v] & ~s_bset[v];
-          s_flag = left != 0;
+#pragma unroll
+        for (int i = 0; i < KW; ++i) {
+          const int w = lane + 32 * i;
+          if (w < W && acc[i]) atomicOr(&s_items[w], acc[i]);
         }
-        __syncthreads();
-        if (!s_flag) break;
+      }
+      __syncthreads();
+      for (int w = tid; w < W; w += nthr) {
+        uint32_t m = s_items[w];
+        s_items[w] = 0;  // ready for the next entry
+        while (m) {
+          const int bb = __ffs(m) - 1;
+          m &= m - 1;
+          const int Bn = tb.item_next[(w << 5) + bb] - g.T;
+          const uint32_t bit = 1u << (Bn & 31);
+          if (!(s_bset[Bn >> 5] & bit)) atomicOr(&s_bset[Bn >> 5], bit);
+        }
       }
       __syncthreads();
       PH_END(3, t_g);

@@ -169,6 +169,18 @@ class WarpWalker {
   int cur_col = -1;
   uint32_t cur_lbl8[8];      // label set of the arrivals being made (all zero = epsilon)
   bool col_labelled = false; // the open column has a labelled arrival (else only epsilon ones)
+  // Checks by region: the span step about to run is the region's last and
+  // the node after it is a gap resolved by the base chart's good masks.  An
+  // end node all of whose lexer states reach that gap by an epsilon edge is
+  // then not closed: the gap's suffix-mode test (good masks include every
+  // completion an item's closure makes, and the gap advances any waiting
+  // item) gives the same answer for its rows as for their closure.
+  bool defer_to_gap = false;
+  // the pending lexeme at lexer state q reaches a following gap by an epsilon edge
+  __device__ bool eps_into_gap(int q) const {
+    const int a = g.dfa_accept[q];
+    return q == 0 || g.dfa_ext[q] || (a >= 0 && g.skip[a]);
+  }
 
   __device__ WarpWalker(const DevGrammar& g_, const LexEntry* t, WWs w, WSh& s, int nm, long long em, int voc)
       : g(g_), table(t), ws(w), sh(s), nmax(nm), emax(em), vocab(voc), W(g_.W), VW(g_.VW) {}
@@ -1038,7 +1050,21 @@ class WarpWalker {
           arrive(ws.g_last[gi], sh.lbl, true);
         }
       }
-      close_column(c, false);
+      bool defer = false;
+      if (EXT && defer_to_gap) {
+        bool all_eps = true;
+        for (int tj = (int)wl_lane(); tj < nt; tj += 32)
+          if (ws.key_q[tj] == ti && !eps_into_gap(ws.f_q[tj])) all_eps = false;
+        defer = __all_sync(0xffffffffu, all_eps);
+      }
+      if (defer) {
+        // rows as they arrived: only their summaries (scatter filters)
+        int o = -1;
+        while ((o = bm_next(sh.touched, o + 1, c + 1)) >= 0) row_scan(row_of(o), sh.vset, sum_of(o));
+        bm_clear(sh.dirty, c + 1);
+      } else {
+        close_column(c, false);
+      }
       finish_column(c);
       if (status) return false;
       if (wl_lane() == 0) ws.f_c[ti] = c;
