@@ -56,6 +56,7 @@ def _load():
             lib.orc_valid.argtypes = [C.c_void_p, i32p, C.c_int, i64p]
             lib.orc_chart_census.argtypes = [C.c_void_p, i32p, C.c_int, i64p, i32p, u8p, C.c_int]
             lib.orc_accepts_terms.argtypes = [C.c_void_p, i32p, C.c_int]
+            lib.orc_graph_accepts_terms.argtypes = [C.c_void_p, i32p, C.c_int, i32p, C.c_int]
             lib.orc_cover_accepts_terms.argtypes = [C.c_void_p, i32p, C.c_int]
             lib.orc_cover_valid.argtypes = [C.c_void_p, i32p, C.c_int]
             lib.orc_validate_batch.argtypes = [C.c_void_p, i32p, C.c_int, C.c_int, i32p, C.c_int,
@@ -168,6 +169,14 @@ class Oracle:
     def accepts_terms(self, terms):
         t = np.ascontiguousarray(terms if len(terms) else [0], np.int32)
         return bool(self._lib.orc_accepts_terms(self.h, _p(t, C.c_int32), len(terms)))
+
+    def graph_accepts_terms(self, x, terms):
+        """Is the terminal sequence a path label of x's partial-output graph
+        (a lexeme sequence compatible with x, gaps reading anything)?"""
+        x = np.ascontiguousarray(x, np.int32)
+        t = np.ascontiguousarray(terms if len(terms) else [0], np.int32)
+        return bool(self._lib.orc_graph_accepts_terms(self.h, _p(x, C.c_int32), len(x), _p(t, C.c_int32),
+                                                       len(terms)))
 
     def cover_accepts_terms(self, terms):
         t = np.ascontiguousarray(terms if len(terms) else [0], np.int32)

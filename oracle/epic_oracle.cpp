@@ -842,6 +842,48 @@ int orc_chart_census(void* h, const int* x, int n, long long* items, int* origin
   return G.n_nodes;
 }
 
+// Is the terminal sequence the label of a path of x's partial-output graph,
+// from its start node to its accept node (epsilon edges free, a gap node
+// reading any terminal on its self-loop)?  The graph's language is C_x of
+// Sec. 3 at the lexeme level, so with orc_accepts_terms this checks a witness
+// completion (Sec. 4.4): a string of L(G) compatible with x.  Forward
+// state-set simulation.
+int orc_graph_accepts_terms(void* h, const int* x, int n, const int* terms, int len) {
+  Grammar& g = ((Oracle*)h)->g;
+  LexMemo memo;
+  Graph G = build_graph(g, std::vector<int>(x, x + n), memo);
+  if (G.dead) return 0;
+  auto eps_close = [&](std::vector<char>& S) {
+    std::vector<int> stack;
+    for (int u = 0; u < G.n_nodes; ++u)
+      if (S[u]) stack.push_back(u);
+    while (!stack.empty()) {
+      int u = stack.back();
+      stack.pop_back();
+      for (auto& e : G.out[u])
+        if (e.first < 0 && !S[e.second]) {
+          S[e.second] = 1;
+          stack.push_back(e.second);
+        }
+    }
+  };
+  std::vector<char> S(G.n_nodes, 0);
+  S[G.start] = 1;
+  eps_close(S);
+  for (int i = 0; i < len; ++i) {
+    std::vector<char> N(G.n_nodes, 0);
+    for (int u = 0; u < G.n_nodes; ++u) {
+      if (!S[u]) continue;
+      if (G.gap[u]) N[u] = 1;  // the gap's self-loop reads any terminal
+      for (auto& e : G.out[u])
+        if (e.first == terms[i]) N[e.second] = 1;
+    }
+    eps_close(N);
+    S.swap(N);
+  }
+  return S[G.accept] ? 1 : 0;
+}
+
 // Earley acceptance of a plain terminal string (a graph that is one path).
 int orc_accepts_terms(void* h, const int* terms, int len) {
   Grammar& g = ((Oracle*)h)->g;

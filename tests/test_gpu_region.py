@@ -117,3 +117,24 @@ def test_clike_full_length_row(cuda):
     assert st['region_checks'] == w.cand.size
     ref = oracle.Oracle(w.grammar, w.vocab).validate_batch(w.x, w.pos, w.cand, nthreads=NTHREADS)
     np.testing.assert_array_equal(got, ref)
+
+
+def test_random_stress_full_length_row(cuda):
+    """random-stress-1024 (400 nonterminals, 1,500 productions, 213 item words)
+    on a whole 1,024-token row: 4 positions x 4 candidates, the row's witness
+    token among them, against the oracle's bits stored by
+    tests/golden/make_stress_golden.py (an oracle chart of a thousand tokens
+    takes up to tens of minutes, too long to run here)."""
+    import json
+    here = os.path.dirname(os.path.abspath(__file__))
+    with open(os.path.join(here, 'golden', 'stress1024_checks.json')) as f:
+        gold = json.load(f)
+    c = gold['case']
+    w = make_workload(c['name'], c['seed'], batch=c['batch'], k=c['k'], K=c['K'])
+    pos = np.array([gold['pos']], np.int32)
+    cand = np.array([gold['cand']], np.int32)
+    assert np.array_equal(pos, w.pos)
+    got, st = run_gpu(w.grammar, w.vocab, w.x, pos, cand, cuda)
+    assert st['overflow'] == 0
+    assert st['region_checks'] == cand.size
+    np.testing.assert_array_equal(got[0], np.array(gold['valid'], np.uint8))

@@ -723,3 +723,52 @@ def test_fallback_invariants(name, seed):
                     y = got_x[b].copy()
                     y[w.pos[b, j]] = w.cand[b, j, c]
                     assert not O.valid(y)
+
+
+# ------------------------------------------------------------------ witness checking
+def test_graph_accepts_unmasked_rows_exactly_their_lexing():
+    """A row without masks has one lexeme sequence (reading 1): the graph's
+    path labels are exactly it (the independent regex-module lexer gives it);
+    dropping, adding or changing one terminal is rejected."""
+    g = expr()
+    vocab = vocab_for(g, ['1+', '(2', '3)', '*(', ' 4', '^-'])
+    O = oracle.Oracle(g, vocab)
+    rng = np.random.default_rng(17)
+    tested = 0
+    for _ in range(300):
+        x = rng.integers(0, len(vocab), int(rng.integers(1, 6))).astype(np.int32)
+        text = b''.join(vocab[t] for t in x).decode()
+        run = lexer_regex_module(g, text, True)
+        if run is None:
+            continue
+        assert O.graph_accepts_terms(x, run), (text, run)
+        if run:
+            assert not O.graph_accepts_terms(x, run[:-1])
+            changed = list(run)
+            changed[0] = (changed[0] + 1) % g.T
+            assert not O.graph_accepts_terms(x, changed)
+        assert not O.graph_accepts_terms(x, list(run) + [0])
+        tested += 1
+    assert tested > 150
+
+
+def test_graph_accepts_matches_gap_regex():
+    """tiny_paren (one-character terminals, spaces skipped): the path labels
+    of a partial output are its fixed runs with any terminal string in each
+    gap -- a regular expression written from the gap model (Sec. 3), checked
+    on every terminal string up to length 5."""
+    import re
+    g = tiny_paren()
+    vocab = [b'(', b')', b'a', b'b', b' ', b'((', b'a)', b' (']
+    O = oracle.Oracle(g, vocab)
+    names = {t.name: i for i, t in enumerate(g.terminals)}
+    sym = {names[c]: c for c in '()ab'}
+    words = [''.join(s) for m in range(6) for s in itertools.product('()ab', repeat=m)]
+    rng = np.random.default_rng(2)
+    for _ in range(60):
+        x = random_partial(rng, len(vocab), int(rng.integers(1, 5)), 0.4)
+        segs, ngaps = _paren_runs(vocab, x)
+        pattern = '.*'.join(re.escape(sg) for sg in segs)
+        for wd in words:
+            terms = [names[c] for c in wd]
+            assert O.graph_accepts_terms(x, terms) == bool(re.fullmatch(pattern, wd)), (x, wd)
