@@ -49,6 +49,8 @@ def parse():
     ap.add_argument('--no-cpu-baseline', action='store_true')
     ap.add_argument('--k', type=int, default=None, help='proposed positions per sequence (sweep)')
     ap.add_argument('--batch', type=int, default=None, help='sequences per batch (smaller cases for profiling)')
+    ap.add_argument('--lazy-lex', type=int, default=None, metavar='CAP',
+                    help='lexing memo filled on use (Alg. 2) with CAP entries instead of the dense table')
     return ap.parse_args()
 
 
@@ -304,7 +306,10 @@ def main():
     from synth import make_workload
     w = make_workload(args.workload, args.seed + rank, k=args.k, batch=args.batch)
     g = epic.Grammar(w.grammar)
-    t = epic.LexTable(g, w.vocab)
+    torch.cuda.synchronize()
+    tb0 = time.perf_counter()
+    t = epic.LexTable(g, w.vocab, lazy_capacity=args.lazy_lex)
+    table_ms = (time.perf_counter() - tb0) * 1e3  # the build synchronizes
     x0 = torch.from_numpy(w.x).to(dev)
     x = x0.clone()
     pos = torch.from_numpy(w.pos).to(dev)
@@ -325,13 +330,13 @@ def main():
         epic.pick_candidates(cand, conf3, valid, tok, conf)
         epic.select_compatible_subset(g, t, xbuf, pos, tok, conf, sel)
         epic.commit(xbuf, pos, tok, sel)
-        epic.fallback_commit(g, t, xbuf, pos, cand, conf3, n_target, sel, filled)
+        epic.fallback_commit(g, t, xbuf, pos, cand, conf3, n_target, sel, filled, valid=valid)
 
     for _ in range(args.warmup):
         x.copy_(x0)
         step(x)
     torch.cuda.synchronize()
-    t.stats(reset=True)
+    st_warm = t.stats(reset=True)  # the warm-up steps, from a cold lexing memo
     # ---- device-timed region: per-step events, L2 flushed before each step
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
            torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
@@ -349,7 +354,7 @@ def main():
             epic.pick_candidates(cand, conf3, valid, tok, conf)
             epic.select_compatible_subset(g, t, x, pos, tok, conf, sel)
             epic.commit(x, pos, tok, sel)
-            epic.fallback_commit(g, t, x, pos, cand, conf3, n_target, sel, filled)
+            epic.fallback_commit(g, t, x, pos, cand, conf3, n_target, sel, filled, valid=valid)
             ev[i][2].record(stream)
             for kname, kms in t.kernel_times().items():  # waits for this step's kernels
                 kern.setdefault(kname, []).append(kms)
@@ -447,6 +452,12 @@ def main():
             'valid_fraction': st['valid'] / max(1, st['checks']), 'overflow': st['overflow'],
             'gpu_launches': int(launches), 'validate_path': 'region' if region else 'walk',
             'commits': commit_sizes,
+            'lex_table': {'kind': 'lazy memo (Alg. 2), %d entries' % args.lazy_lex if args.lazy_lex else 'dense',
+                          'build_ms': table_ms,
+                          'memo_hit_rate_warmup': ((1.0 - st_warm['lex_misses'] / st_warm['lex_lookups'])
+                                                   if st_warm['lex_lookups'] else None),
+                          'memo_hit_rate_timed': (1.0 - st['lex_misses'] / st['lex_lookups']) if st['lex_lookups'] else None,
+                          'lookups_per_step': st['lex_lookups'] / max(1, args.steps)},
             'e2e': {'value': total_checks / (e2e_step / 1e3), 'unit': 'checks/s', 'h2d_bytes_per_step': int(h2d),
                     'd2h_bytes_per_step': int(d2h)},
             'roofline': roof, 'clocks': clk.summary()}

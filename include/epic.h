@@ -109,11 +109,28 @@ int32_t epic_grammar_lexer_states(const epic_grammar* g);
 epic_status epic_lexer_table_build(const epic_grammar* g, const int32_t* tok_off,
                                    const uint8_t* tok_bytes, int32_t vocab, void* cuda_stream,
                                    epic_lexer_table** out);
+/*
+ * The same lexing table built lazily (Alg. 2: lexing results are memoized as
+ * they are first needed, not precomputed): no dense [vocab][states] table is
+ * built; a device hash table of `capacity` entries (rounded up to a power of
+ * two, at most 2^30) keyed by (token, lexer state) is filled by the walks,
+ * each entry computed by the transducer above on its first lookup.  Every
+ * call gives the same results as with the dense table.  A lookup that finds
+ * no free slot within 64 probes computes its entry without storing it
+ * (stats.lex_uncached).  Counters: stats.lex_lookups, stats.lex_misses (the
+ * memo's hit rate is 1 - misses / lookups).  Errors as epic_lexer_table_build,
+ * plus EPIC_ERR_CAPACITY when vocab x states does not fit 32-bit keys.
+ * epic_lexer_table_copy is not available for lazy tables.  Synchronous.
+ */
+epic_status epic_lexer_table_build_lazy(const epic_grammar* g, const int32_t* tok_off,
+                                        const uint8_t* tok_bytes, int32_t vocab, int64_t capacity,
+                                        void* cuda_stream, epic_lexer_table** out);
 void epic_lexer_table_destroy(epic_lexer_table* t);
 
 /*
  * Copy lex-table entries of tokens [first_token, first_token + count) to host
- * memory (synchronous; for inspection and tests).  Entry (t, q) is 16 bytes:
+ * memory (synchronous; an inspection aid of the table of Sec. 4.1, used by
+ * the tests; dense tables only).  Entry (t, q) is 16 bytes:
  * uint16 end state (0xFFFF = DEAD), uint8 run length, uint8 terminals[13].
  * host_out must hold count * epic_grammar_lexer_states(g) * 16 bytes.
  */
@@ -141,8 +158,11 @@ epic_status epic_lexer_table_copy(const epic_lexer_table* t, int32_t first_token
  * batch has more checks than resident walks, one forward chart of x per
  * sequence (with its graph and good-item masks) and one warp per check
  * walking only the candidate's region (stats.region_checks counts these).
- * The library's device workspaces grow on demand (the per-sequence charts
- * up to EPIC_SEQ_WORKSPACE_MB, default 80 GiB); a failed allocation returns
+ * The library's device workspaces grow on demand, each up to a share of the
+ * GPU's memory (per-sequence charts 30 %, per-warp walks 25 %, block walks of
+ * selection 25 %, never more than is free; EPIC_SEQ_WORKSPACE_MB,
+ * EPIC_WARP_WORKSPACE_MB and EPIC_WORKSPACE_MB override, in MiB).  Smaller
+ * budgets run fewer walks at a time; a failed allocation returns
  * EPIC_ERR_OOM.  A sequence whose chart does not fit walks its checks whole.
  */
 epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t,
@@ -233,9 +253,14 @@ epic_status epic_commit(int32_t* d_x, int32_t B, int32_t n, const int32_t* d_pos
  * d_x [B][n] int32, updated in place (call after epic_commit of the selected
  * batch); d_pos [B][k], d_cand [B][k][K], d_cand_conf [B][k][K] float32 as
  * for epic_pick_candidates; d_n_target [B] int32 = n_t, the commits wanted
- * in this step; d_selected [B][k] (1 = in B) or NULL for |B| = 0; output
- * d_filled [B][k] int32: the token this call committed at slot j, else -1.
- * One CTA per sequence; each test is a whole-graph walk of x (+) c.
+ * in this step; d_selected [B][k] (1 = in B) or NULL for |B| = 0;
+ * d_valid [B][k][K] or NULL: epic_validate_batch's bits for the same
+ * candidates on x before the selected batch was committed -- a candidate
+ * whose bit is 0 is rejected without a test (it would fail it: a partial
+ * output that is not completable stays so after more commits, App. D); the
+ * result is the same with or without it.  Output d_filled [B][k] int32: the
+ * token this call committed at slot j, else -1.  One CTA per sequence; each
+ * test is a whole-graph walk of x (+) c.
  * Errors: EPIC_ERR_INVALID_ARG (NULL pointers, sizes < 0),
  * EPIC_ERR_CAPACITY when k K > 4096.  A NaN confidence or a position out of
  * range leaves that sequence unchanged (stats.bad_inputs); a test that hits
@@ -245,7 +270,26 @@ epic_status epic_commit(int32_t* d_x, int32_t B, int32_t n, const int32_t* d_pos
 epic_status epic_fallback_commit(const epic_grammar* g, const epic_lexer_table* t, int32_t* d_x, int32_t B,
                                  int32_t n, const int32_t* d_pos, int32_t k, const int32_t* d_cand,
                                  const float* d_cand_conf, int32_t K, const int32_t* d_n_target,
-                                 const uint8_t* d_selected, int32_t* d_filled, void* cuda_stream);
+                                 const uint8_t* d_selected, const uint8_t* d_valid, int32_t* d_filled,
+                                 void* cuda_stream);
+
+/*
+ * Witness extraction for failure recovery (Sec. 4.4): for each row of d_x
+ * [B][n], one completion -- a lexeme sequence of L(G) that the partial output
+ * allows (C_x of Sec. 3) -- read off the row's forward Earley chart by a
+ * top-down walk of the accepting item's derivation.  Output d_terms [B][cap]
+ * int32: the terminal ids in order, each with bit 16 set when a mask run (a
+ * gap) produces it (the recovery fills those runs), the rest being the
+ * lexemes of the fixed text; d_len [B] int32: the length, -1 when the row is
+ * not completable (no witness exists), -2 when its chart, the capacity cap or
+ * the search bound was exceeded (stats.witness_failures counts searches that
+ * found no derivation).  A nonterminal that a gap derives is written as one
+ * of its shortest terminal strings.  Runs the forward charts of
+ * epic_validate_batch's checks by region, then one warp per row.  Errors:
+ * EPIC_ERR_INVALID_ARG (NULL pointers, sizes < 0, cap < 1).  Asynchronous.
+ */
+epic_status epic_extract_witness(const epic_grammar* g, const epic_lexer_table* t, const int32_t* d_x, int32_t B,
+                                 int32_t n, int32_t* d_terms, int32_t cap, int32_t* d_len, void* cuda_stream);
 
 /* Device counters accumulated since the object was created (or reset). */
 typedef struct {
@@ -263,6 +307,10 @@ typedef struct {
   uint64_t validate_kernels; /* kernel launches made by epic_validate_batch*  */
   uint64_t fallback_checks;  /* exact tests of the rejection fallback         */
   uint64_t fallback_commits; /* candidates it committed                       */
+  uint64_t lex_lookups;      /* (token, lexer state) lookups of span lexing   */
+  uint64_t lex_misses;       /* lazy tables: entries computed on first use    */
+  uint64_t lex_uncached;     /* lazy tables: computed without a free slot     */
+  uint64_t witness_failures; /* witness searches that found no derivation     */
 } epic_stats;
 
 /* Copy the counters (synchronizes the lexer table's last stream); out_bytes

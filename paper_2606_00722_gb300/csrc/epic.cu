@@ -4,6 +4,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <functional>
 #include <mutex>
 #include <new>
 #include <stdexcept>
@@ -28,39 +29,9 @@ __global__ void k_lex_table(const int32_t* __restrict__ tok_off, const uint8_t* 
   long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (long long)vocab * Q) return;
   int t = (int)(idx / Q), q = (int)(idx % Q);
-  LexEntry e;
-  uint32_t* raw = reinterpret_cast<uint32_t*>(&e);
-  raw[0] = raw[1] = raw[2] = raw[3] = 0;
-  int s = q, len = 0;
-  bool dead = false;
-  for (int i = tok_off[t]; i < tok_off[t + 1]; ++i) {
-    int c = bytes[i];
-    int nx = dfa_next[s * 256 + c];
-    if (nx >= 0) {
-      s = nx;
-      continue;
-    }
-    int a = dfa_acc[s];  // q0 never accepts (no terminal matches epsilon)
-    if (a < 0) {
-      dead = true;
-      break;
-    }
-    if (!skip[a]) {
-      if (len >= 13) {
-        atomicExch(overflow, 1);
-        dead = true;
-        break;
-      }
-      e.term[len++] = (uint8_t)a;
-    }
-    s = dfa_next[c];  // restart from q0 on c
-    if (s < 0) {
-      dead = true;
-      break;
-    }
-  }
-  e.end = dead ? 0xFFFF : (uint16_t)s;
-  e.len = dead ? 0 : (uint8_t)len;
+  bool ovf = false;
+  const LexEntry e = lex_transduce(bytes, tok_off[t], tok_off[t + 1], q, dfa_next, dfa_acc, skip, &ovf);
+  if (ovf) atomicExch(overflow, 1);
   table[idx] = e;
 }
 
@@ -109,7 +80,15 @@ struct epic_grammar {
 struct epic_lexer_table {
   const epic_grammar* g = nullptr;
   int vocab = 0;
-  LexEntry* d_table = nullptr;
+  LexEntry* d_table = nullptr;  // dense tables; null for lazy ones
+  // the grammar's device tables with this table's lazy memo (keys null: dense)
+  DevGrammar dgl{};
+  uint32_t* d_lz_keys = nullptr;  // lazy memo (Alg. 2's cache filled on use)
+  uint32_t* d_lz_ready = nullptr;
+  LexEntry* d_lz_vals = nullptr;
+  int32_t* d_lz_off = nullptr;
+  uint8_t* d_lz_bytes = nullptr;
+  long long lz_cap = 0;
   char* d_ws = nullptr;
   size_t ws_bytes = 0;
   WsDims dims{};
@@ -121,6 +100,8 @@ struct epic_lexer_table {
   char* d_seq = nullptr;     // per-sequence forward charts (region checks)
   size_t seq_bytes = 0;
   int32_t* d_regs = nullptr; // per-warp tables of region checks
+  char* d_wit = nullptr;     // witness extraction: goals and stack per sequence
+  size_t wit_bytes = 0;
   size_t regs_bytes = 0;
   int spec_cap = 0;
   char* d_wws = nullptr;   // warp-walk workspace
@@ -169,21 +150,33 @@ int sm_count() {
   return n > 0 ? n : 1;
 }
 
+// Default budget of one device workspace: a share of the GPU's memory, and no
+// more than is free now plus what the workspace already holds (it is freed
+// before it grows), less 1 GiB of headroom.  An environment variable (MiB)
+// overrides.  The three workspaces (per-sequence charts 30 %, warp walks
+// 25 %, block walks 25 %) leave a fifth of the GPU to the caller.
+size_t workspace_budget(const char* env, double share, size_t held) {
+  if (const char* e = getenv(env)) return strtoull(e, nullptr, 10) << 20;
+  size_t free_b = 0, total_b = 0;
+  if (cudaMemGetInfo(&free_b, &total_b) != cudaSuccess) return (size_t)4096 << 20;
+  const size_t headroom = (size_t)1 << 30;
+  size_t avail = free_b + held > headroom ? free_b + held - headroom : 0;
+  return std::min((size_t)(share * (double)total_b), avail);
+}
+
 // Block-walk workspace of selection and the fallback: every CTA gets room
 // for one whole chart of a row (4,096 columns, 640 n entries, as the
 // per-sequence forward charts; EPIC_ENTRIES_PER_CTA overrides), and as many
-// CTAs as asked run if their workspaces fit EPIC_WORKSPACE_MB (default
-// 32 GiB), else fewer (the kernels loop over their sequences).
+// CTAs as asked run if their workspaces fit EPIC_WORKSPACE_MB (default a
+// quarter of the GPU), else fewer (the kernels loop over their sequences).
 epic_status ensure_workspace(epic_lexer_table* t, int want_ctas, int n, cudaStream_t st) {
   const epic_grammar* g = t->g;
-  size_t budget_mb = 32768;
-  if (const char* e = getenv("EPIC_WORKSPACE_MB")) budget_mb = strtoull(e, nullptr, 10);
   int W = g->dg.W, VW = g->dg.VW, FW = g->dg.FW;
   WsDims d;
   d.nmax = kMaxCols;
   d.emax = std::max<long long>(4096, 640ll * std::max(1, n));
   if (const char* e = getenv("EPIC_ENTRIES_PER_CTA")) d.emax = std::max<long long>(64, atoll(e));
-  const size_t budget = budget_mb << 20;
+  const size_t budget = workspace_budget("EPIC_WORKSPACE_MB", 0.25, t->d_ws ? t->ws_bytes : 0);
   size_t per = ws_bytes_per_cta(d, W, VW, FW);
   while (per > budget && d.emax > 4096) {  // not even one CTA fits: smaller charts
     d.emax = d.emax * 3 / 4;
@@ -214,15 +207,14 @@ epic_status ensure_workspace(epic_lexer_table* t, int want_ctas, int n, cudaStre
 
 // Warp-walk workspace: columns <= min(4096, 8 n + 256) per walk; entries
 // per walk EPIC_ENTRIES_PER_WALK (default 256 n); warps cut down until the
-// total fits EPIC_WARP_WORKSPACE_MB (default 6144).
+// total fits EPIC_WARP_WORKSPACE_MB (default a quarter of the GPU).
 epic_status ensure_wworkspace(epic_lexer_table* t, long long checks, int n, cudaStream_t st) {
   const epic_grammar* g = t->g;
   int W = g->dg.W, VW = g->dg.VW;
   int nmax = std::min(kWCols, 8 * n + 256);
   long long emax = 256ll * std::max(1, n);
   if (const char* e = getenv("EPIC_ENTRIES_PER_WALK")) emax = atoll(e);
-  size_t budget = (size_t)6144 << 20;
-  if (const char* e = getenv("EPIC_WARP_WORKSPACE_MB")) budget = strtoull(e, nullptr, 10) << 20;
+  const size_t budget = workspace_budget("EPIC_WARP_WORKSPACE_MB", 0.25, t->d_wws ? t->wws_bytes : 0);
   size_t per = wbytes_per_warp(nmax, emax, W, VW);
   long long warps = std::min<long long>(checks, (long long)sm_count() * 2 * kWarpsPerCta);
   warps = std::max<long long>(kWarpsPerCta, (warps + kWarpsPerCta - 1) / kWarpsPerCta * kWarpsPerCta);
@@ -277,16 +269,16 @@ epic_status grow(epic_lexer_table* t, char** buf, size_t* have, size_t need) {
   return EPIC_OK;
 }
 
-// Region checks: forward chart and good masks per sequence, then one warp per
-// check.  Capacities: EPIC_SEQ_ENTRIES (default 400 n) chart entries per
-// sequence, EPIC_SEQ_WORKSPACE_MB (default 81920) in total; checks of a
-// sequence whose chart does not fit walk their whole graph instead.
-epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const int32_t* d_x, int B, int n,
-                            const int32_t* d_pos, int k, const int32_t* d_cand, int K, uint8_t* d_valid,
-                            cudaStream_t st) {
-  const DevGrammar& dg = g->dg;
-  long long total = (long long)B * k * K;
-  SeqPack sp;
+// Checks by region, steps 1-2 (also the start of witness extraction): the
+// per-sequence arena (EPIC_SEQ_ENTRIES, default 640 n chart entries per
+// sequence; EPIC_SEQ_WORKSPACE_MB, default 30 % of the GPU, caps the batch:
+// a sequence whose chart does not fit its arena has its checks walk the
+// whole graph instead), the forward charts and the good masks with their
+// indexes.
+epic_status region_prepare(const epic_grammar* g, epic_lexer_table* t, const int32_t* d_x, int B, int n, SeqPack& sp,
+                           cudaStream_t st) {
+  (void)g;
+  const DevGrammar& dg = t->dgl;
   sp.nmax = std::min(kMaxCols, 8 * n + 256);
   sp.n = n;
   sp.W = dg.W;
@@ -294,47 +286,12 @@ epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const in
   sp.edge_cap = 32 * sp.nmax;
   sp.emax = 640ll * n;
   if (const char* e = getenv("EPIC_SEQ_ENTRIES")) sp.emax = atoll(e);
-  size_t budget = (size_t)81920 << 20;
-  if (const char* e = getenv("EPIC_SEQ_WORKSPACE_MB")) budget = strtoull(e, nullptr, 10) << 20;
+  const size_t budget = workspace_budget("EPIC_SEQ_WORKSPACE_MB", 0.30, t->d_seq ? t->seq_bytes : 0);
   while (sp.emax > 4096 && sp.bytes() * (size_t)B > budget) sp.emax = sp.emax * 3 / 4;
   sp.per_seq = sp.bytes();
   epic_status s = grow(t, &t->d_seq, &t->seq_bytes, sp.per_seq * (size_t)B);
   if (s != EPIC_OK) return s;
   sp.base = t->d_seq;
-  // per-warp workspace of the checks: own columns after the chart's
-  WPack wp;
-  wp.nmax = kWCols;
-  // own entries: the region's columns and the rows carried after it
-  wp.emax = std::max(8192ll, 64ll * n);
-  if (const char* e = getenv("EPIC_ENTRIES_PER_WALK")) wp.emax = atoll(e);
-  wp.W = dg.W;
-  wp.VW = dg.VW;
-  wp.per_warp = wbytes_per_warp(wp.nmax, wp.emax, wp.W, wp.VW);
-  size_t wbudget = (size_t)6144 << 20;
-  if (const char* e = getenv("EPIC_WARP_WORKSPACE_MB")) wbudget = strtoull(e, nullptr, 10) << 20;
-  long long warps = std::min<long long>(total, (long long)sm_count() * 2 * kWarpsPerCta);
-  warps = std::max<long long>(1, warps);
-  while (warps > 1 && wp.per_warp * (size_t)warps > wbudget) warps = warps * 3 / 4;
-  size_t wneed = wp.per_warp * (size_t)warps;
-  if (!t->d_wws || t->wws_bytes < wneed || t->wnmax != wp.nmax || t->wemax != wp.emax) {
-    if (t->d_wws) {
-      cudaStreamSynchronize(t->last);
-      cudaFree(t->d_wws);
-      t->d_wws = nullptr;
-    }
-    if (cudaMalloc(&t->d_wws, wneed) != cudaSuccess) {
-      t->d_wws = nullptr;
-      return EPIC_ERR_OOM;
-    }
-    // the global stage starts at zero; walks return it zeroed
-    if (cudaMemsetAsync(t->d_wws, 0, wneed, st) != cudaSuccess) return EPIC_ERR_CUDA;
-    t->wws_bytes = wneed;
-    t->wnmax = wp.nmax;
-    t->wemax = wp.emax;
-  }
-  wp.base = t->d_wws;
-  s = grow(t, (char**)&t->d_regs, &t->regs_bytes, (size_t)warps * 3 * wp.nmax * 4);
-  if (s != EPIC_OK) return s;
   t->last = st;
   const size_t smem_cap = 190 * 1024;
   const int rmax = 256;
@@ -368,6 +325,55 @@ epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const in
   mark(t, 1, st);
   launch_good(B, st, dg, B, sp);
   mark(t, 2, st);
+  return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
+}
+
+epic_status validate_region(const epic_grammar* g, epic_lexer_table* t, const int32_t* d_x, int B, int n,
+                            const int32_t* d_pos, int k, const int32_t* d_cand, int K, uint8_t* d_valid,
+                            cudaStream_t st) {
+  const DevGrammar& dg = t->dgl;
+  long long total = (long long)B * k * K;
+  // per-warp workspace of the checks: own columns after the chart's
+  WPack wp;
+  wp.nmax = kWCols;
+  // own entries: the region's columns and the rows carried after it
+  wp.emax = std::max(8192ll, 64ll * n);
+  if (const char* e = getenv("EPIC_ENTRIES_PER_WALK")) wp.emax = atoll(e);
+  wp.W = dg.W;
+  wp.VW = dg.VW;
+  wp.per_warp = wbytes_per_warp(wp.nmax, wp.emax, wp.W, wp.VW);
+  const size_t wbudget = workspace_budget("EPIC_WARP_WORKSPACE_MB", 0.25, t->d_wws ? t->wws_bytes : 0);
+  long long warps = std::min<long long>(total, (long long)sm_count() * 2 * kWarpsPerCta);
+  warps = std::max<long long>(1, warps);
+  warps = std::max<long long>(1, std::min<long long>(warps, (long long)(wbudget / wp.per_warp)));
+  size_t wneed = wp.per_warp * (size_t)warps;
+  if (!t->d_wws || t->wws_bytes < wneed || t->wnmax != wp.nmax || t->wemax != wp.emax) {
+    if (t->d_wws) {
+      cudaStreamSynchronize(t->last);
+      cudaFree(t->d_wws);
+      t->d_wws = nullptr;
+    }
+    if (cudaMalloc(&t->d_wws, wneed) != cudaSuccess) {
+      t->d_wws = nullptr;
+      return EPIC_ERR_OOM;
+    }
+    // the global stage starts at zero; walks return it zeroed
+    if (cudaMemsetAsync(t->d_wws, 0, wneed, st) != cudaSuccess) return EPIC_ERR_CUDA;
+    t->wws_bytes = wneed;
+    t->wnmax = wp.nmax;
+    t->wemax = wp.emax;
+  }
+  wp.base = t->d_wws;
+  epic_status s = grow(t, (char**)&t->d_regs, &t->regs_bytes, (size_t)warps * 3 * wp.nmax * 4);
+  if (s != EPIC_OK) return s;
+  t->last = st;
+  const size_t smem_cap = 190 * 1024;
+  const int rmax = 256;
+  bool sm = dg.W <= 32;
+  // 1-2. forward charts and good masks
+  SeqPack sp;
+  s = region_prepare(g, t, d_x, B, n, sp, st);
+  if (s != EPIC_OK) return s;
   t->n_region += total;
   t->n_vkernels += 3;
   // 3. checks
@@ -555,6 +561,72 @@ epic_status epic_grammar_create(const epic_grammar_desc* desc, epic_grammar** ou
     }
     up(pw, &d.adv_pow);
   }
+  {
+    // witness extraction tables: complete items by left side, and a shortest
+    // terminal string of every nonterminal (fixpoint of the shortest yield
+    // length; a production is chosen only when it strictly shortens, so the
+    // choices form no cycle and expand to finite strings)
+    const int V = G.V, T = G.T;
+    const int P2 = (int)G.lhs.size();
+    std::vector<int32_t> coff(V + 1, 0), citems;
+    for (int p = 0; p < P2; ++p)
+      if (G.lhs[p] >= 0) ++coff[G.lhs[p] + 1];
+    for (int v = 0; v < V; ++v) coff[v + 1] += coff[v];
+    citems.assign(coff[V], 0);
+    std::vector<int32_t> cur(coff.begin(), coff.end() - 1);
+    for (int p = 0; p < P2; ++p)
+      if (G.lhs[p] >= 0) citems[cur[G.lhs[p]]++] = G.item_base[p] + (G.rhs_off[p + 1] - G.rhs_off[p]);
+    const long long INF = 1ll << 40;
+    std::vector<long long> len(V, INF);
+    std::vector<int> best(V, -1);
+    for (bool changed = true; changed;) {
+      changed = false;
+      for (int p = 0; p < P2; ++p) {
+        if (G.lhs[p] < 0) continue;
+        long long L = 0;
+        for (int i = G.rhs_off[p]; i < G.rhs_off[p + 1] && L < INF; ++i) {
+          const int X = G.rhs[i];
+          L += X < T ? 1 : len[X - T];
+        }
+        if (L < len[G.lhs[p]]) {
+          len[G.lhs[p]] = L;
+          best[G.lhs[p]] = p;
+          changed = true;
+        }
+      }
+    }
+    std::vector<int32_t> yoff(V + 1, 0), ys;
+    std::vector<std::vector<int32_t>> memo(V);
+    std::vector<char> done(V, 0);
+    std::function<void(int, std::vector<int32_t>&)> expand = [&](int A, std::vector<int32_t>& out) {
+      if (done[A]) {
+        out.insert(out.end(), memo[A].begin(), memo[A].end());
+        return;
+      }
+      std::vector<int32_t> mine;
+      const int p = best[A];
+      if (p >= 0 && mine.size() < 4096)
+        for (int i = G.rhs_off[p]; i < G.rhs_off[p + 1]; ++i) {
+          const int X = G.rhs[i];
+          if (X < T) mine.push_back(X);
+          else expand(X - T, mine);
+        }
+      if (mine.size() > 4096) mine.resize(4096);
+      memo[A] = mine;
+      done[A] = 1;
+      out.insert(out.end(), mine.begin(), mine.end());
+    };
+    for (int v = 0; v < V; ++v) {
+      std::vector<int32_t> y;
+      if (len[v] < INF) expand(v, y);
+      yoff[v + 1] = yoff[v] + (int)y.size();
+      ys.insert(ys.end(), y.begin(), y.end());
+    }
+    up(coff, &d.nt_comp_off);
+    up(citems, &d.nt_comp);
+    up(yoff, &d.ny_off);
+    up(ys, &d.ny);
+  }
   d.FS = g->cov.FS;
   d.FW = g->cov.FW;
   d.cov_start = g->cov.start;
@@ -593,6 +665,8 @@ epic_status epic_lexer_table_build(const epic_grammar* g, const int32_t* tok_off
   t->g = g;
   t->vocab = vocab;
   t->last = st;
+  t->dgl = g->dg;
+  t->dgl.lazy = LazyLex{};
   int Q = g->dg.Q;
   size_t nbytes = (size_t)tok_off[vocab];
   int32_t* d_off = nullptr;
@@ -629,6 +703,62 @@ epic_status epic_lexer_table_build(const epic_grammar* g, const int32_t* tok_off
     epic_lexer_table_destroy(t);
     return res;
   }
+  t->dgl.lazy.stats = t->d_stats + S_LEX_LOOKUPS;  // lookups are counted for dense tables too
+  *out = t;
+  return EPIC_OK;
+}
+
+epic_status epic_lexer_table_build_lazy(const epic_grammar* g, const int32_t* tok_off, const uint8_t* tok_bytes,
+                                        int32_t vocab, int64_t capacity, void* cuda_stream, epic_lexer_table** out) {
+  if (!g || !tok_off || !out || vocab <= 0 || capacity < 1) return EPIC_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (tok_off[0] != 0) return EPIC_ERR_INVALID_ARG;
+  for (int t = 0; t < vocab; ++t) {
+    int L = tok_off[t + 1] - tok_off[t];
+    if (L < 1 || L > 64) return EPIC_ERR_INVALID_ARG;
+  }
+  if (!tok_bytes) return EPIC_ERR_INVALID_ARG;
+  // the key token * Q + state + 1 must fit 32 bits
+  if ((unsigned long long)vocab * (unsigned long long)g->dg.Q >= 0xFFFFFFFFull) return EPIC_ERR_CAPACITY;
+  long long cap = 1;
+  while (cap < capacity) cap <<= 1;
+  if (cap > (1ll << 30)) return EPIC_ERR_CAPACITY;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  epic_lexer_table* t = new (std::nothrow) epic_lexer_table();
+  if (!t) return EPIC_ERR_OOM;
+  t->g = g;
+  t->vocab = vocab;
+  t->last = st;
+  t->lz_cap = cap;
+  size_t nbytes = (size_t)tok_off[vocab];
+  epic_status res = EPIC_OK;
+  if (cudaMalloc(&t->d_lz_keys, (size_t)cap * 4) != cudaSuccess ||
+      cudaMalloc(&t->d_lz_ready, (size_t)cap * 4) != cudaSuccess ||
+      cudaMalloc(&t->d_lz_vals, (size_t)cap * sizeof(LexEntry)) != cudaSuccess ||
+      cudaMalloc(&t->d_lz_off, (size_t)(vocab + 1) * 4) != cudaSuccess ||
+      cudaMalloc(&t->d_lz_bytes, nbytes) != cudaSuccess || cudaMalloc(&t->d_stats, S_N * 8) != cudaSuccess ||
+      cudaMalloc(&t->d_counter, 8) != cudaSuccess)
+    res = EPIC_ERR_OOM;
+  if (res == EPIC_OK) {
+    cudaMemcpyAsync(t->d_lz_off, tok_off, (size_t)(vocab + 1) * 4, cudaMemcpyHostToDevice, st);
+    cudaMemcpyAsync(t->d_lz_bytes, tok_bytes, nbytes, cudaMemcpyHostToDevice, st);
+    cudaMemsetAsync(t->d_lz_keys, 0, (size_t)cap * 4, st);
+    cudaMemsetAsync(t->d_lz_ready, 0, (size_t)cap * 4, st);
+    cudaMemsetAsync(t->d_stats, 0, S_N * 8, st);
+    if (cudaGetLastError() != cudaSuccess || cudaStreamSynchronize(st) != cudaSuccess) res = EPIC_ERR_CUDA;
+  }
+  if (res != EPIC_OK) {
+    epic_lexer_table_destroy(t);
+    return res;
+  }
+  t->dgl = g->dg;
+  t->dgl.lazy.keys = t->d_lz_keys;
+  t->dgl.lazy.ready = t->d_lz_ready;
+  t->dgl.lazy.vals = t->d_lz_vals;
+  t->dgl.lazy.mask = (uint32_t)(cap - 1);
+  t->dgl.lazy.tok_off = t->d_lz_off;
+  t->dgl.lazy.tok_bytes = t->d_lz_bytes;
+  t->dgl.lazy.stats = t->d_stats + S_LEX_LOOKUPS;
   *out = t;
   return EPIC_OK;
 }
@@ -642,8 +772,14 @@ void epic_lexer_table_destroy(epic_lexer_table* t) {
   cudaFree(t->d_spec);
   cudaFree(t->d_seq);
   cudaFree(t->d_regs);
+  cudaFree(t->d_wit);
   cudaFree(t->d_stats);
   cudaFree(t->d_counter);
+  cudaFree(t->d_lz_keys);
+  cudaFree(t->d_lz_ready);
+  cudaFree(t->d_lz_vals);
+  cudaFree(t->d_lz_off);
+  cudaFree(t->d_lz_bytes);
   for (cudaEvent_t e : t->kev)
     if (e) cudaEventDestroy(e);
   for (cudaEvent_t e : t->sev)
@@ -653,7 +789,8 @@ void epic_lexer_table_destroy(epic_lexer_table* t) {
 
 epic_status epic_lexer_table_copy(const epic_lexer_table* t, int32_t first_token, int32_t count, void* host_out,
                                   size_t out_bytes) {
-  if (!t || !host_out || first_token < 0 || count < 0 || first_token + count > t->vocab) return EPIC_ERR_INVALID_ARG;
+  if (!t || !host_out || first_token < 0 || count < 0 || first_token + count > t->vocab || !t->d_table)
+    return EPIC_ERR_INVALID_ARG;
   size_t Q = (size_t)t->g->dg.Q;
   size_t bytes = (size_t)count * Q * sizeof(LexEntry);
   if (out_bytes < bytes) return EPIC_ERR_INVALID_ARG;
@@ -689,7 +826,7 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
   const size_t smem_cap = 190 * 1024;  // + 27 KB static per CTA <= 227 KB
   const int rmax = 256;
   size_t per = smem_per_warp(wp.nmax, rmax, wp.W, wp.VW);
-  const DevGrammar& dg = g->dg;
+  const DevGrammar& dg = t->dgl;
   size_t gt = gtab_bytes(dg.T, dg.V, dg.W, dg.D, dg.Q);
   int gsm = (gt + 4 * per <= smem_cap) ? 1 : 0;  // tables in shared memory if 4 warps still fit
   int wpc = (int)std::min<size_t>(kWarpsPerCta, (smem_cap - (gsm ? gt : 0)) / per);
@@ -707,10 +844,10 @@ epic_status epic_validate_batch(const epic_grammar* g, const epic_lexer_table* t
     size_t dyn = per * wpc + (gsm ? gt : 0);
     int blocks = (t->wwarps + wpc - 1) / wpc;
     if ((size_t)blocks * wpc > (size_t)t->wwarps) blocks = t->wwarps / wpc;
-    launch_validate_warp(true, blocks, 32 * wpc, dyn, st, g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K,
+    launch_validate_warp(true, blocks, 32 * wpc, dyn, st, t->dgl, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand, K,
                          total, d_valid, wp, rmax, gsm, t->d_counter, t->d_stats);
   } else {
-    launch_validate_warp(false, t->wwarps / kWarpsPerCta, 32 * kWarpsPerCta, 0, st, g->dg, t->d_table, t->vocab, d_x,
+    launch_validate_warp(false, t->wwarps / kWarpsPerCta, 32 * kWarpsPerCta, 0, st, t->dgl, t->d_table, t->vocab, d_x,
                          n, d_pos, k, d_cand, K, total, d_valid, wp, 0, 0, t->d_counter, t->d_stats);
   }
   mark(t, 1, st);
@@ -810,7 +947,7 @@ epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_
     int per_cta = (int)std::min<long long>(wpc, warps);
     int blocks = (int)(warps / per_cta);
     size_t dyn = sper * per_cta;
-    launch_validate_warp(true, blocks, 32 * per_cta, dyn, st, g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand,
+    launch_validate_warp(true, blocks, 32 * per_cta, dyn, st, t->dgl, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand,
                          K, total, d_valid, wp, rmax, 0, counter, t->d_stats);
   } else {
     // the global stage and its completed-NT sets must start at zero
@@ -818,7 +955,7 @@ epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_
     int per_cta = (int)std::min<long long>(kWarpsPerCta, warps);
     int blocks = (int)(warps / per_cta);
     if (cudaMemsetAsync(wp.base, 0, wp.per_warp * (size_t)blocks * per_cta, st) != cudaSuccess) return EPIC_ERR_CUDA;
-    launch_validate_warp(false, blocks, 32 * per_cta, 0, st, g->dg, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand,
+    launch_validate_warp(false, blocks, 32 * per_cta, 0, st, t->dgl, t->d_table, t->vocab, d_x, n, d_pos, k, d_cand,
                          K, total, d_valid, wp, 0, 0, counter, t->d_stats);
   }
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
@@ -858,11 +995,11 @@ epic_status epic_select_compatible_subset(const epic_grammar* g, const epic_lexe
   }
   t->last = st;
   mark_event(&t->sev[0], st);
-  launch_select_spec(std::min(2 * B, t->ctas), st, g->dg, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_tok,
+  launch_select_spec(std::min(2 * B, t->ctas), st, t->dgl, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_tok,
                      t->d_spec, pack_of(t));
   mark_event(&t->sev[1], st);
   int ctas = std::min(B, t->ctas);
-  launch_select(ctas, st, g->dg, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_tok, d_conf, d_selected, pack_of(t),
+  launch_select(ctas, st, t->dgl, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_tok, d_conf, d_selected, pack_of(t),
                 t->d_spec, t->d_stats);
   mark_event(&t->sev[2], st);
   t->sel_timed = t->sev[0] && t->sev[1] && t->sev[2];
@@ -872,7 +1009,8 @@ epic_status epic_select_compatible_subset(const epic_grammar* g, const epic_lexe
 epic_status epic_fallback_commit(const epic_grammar* g, const epic_lexer_table* tc, int32_t* d_x, int32_t B,
                                  int32_t n, const int32_t* d_pos, int32_t k, const int32_t* d_cand,
                                  const float* d_cand_conf, int32_t K, const int32_t* d_n_target,
-                                 const uint8_t* d_selected, int32_t* d_filled, void* cuda_stream) {
+                                 const uint8_t* d_selected, const uint8_t* d_valid, int32_t* d_filled,
+                                 void* cuda_stream) {
   epic_lexer_table* t = const_cast<epic_lexer_table*>(tc);
   if (!g || !t || t->g != g || B < 0 || n < 0 || k < 0 || K < 0) return EPIC_ERR_INVALID_ARG;
   if ((long long)B * k == 0) return EPIC_OK;
@@ -883,8 +1021,25 @@ epic_status epic_fallback_commit(const epic_grammar* g, const epic_lexer_table* 
   epic_status s = ensure_workspace(t, std::min(B, sm_count() * 2), n, st);
   if (s != EPIC_OK) return s;
   t->last = st;
-  launch_fallback(std::min(B, t->ctas), st, g->dg, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_cand, d_cand_conf, K,
-                  d_n_target, d_selected, d_filled, pack_of(t), t->d_stats);
+  launch_fallback(std::min(B, t->ctas), st, t->dgl, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_cand, d_cand_conf, K,
+                  d_n_target, d_selected, d_valid, d_filled, pack_of(t), t->d_stats);
+  return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
+}
+
+epic_status epic_extract_witness(const epic_grammar* g, const epic_lexer_table* tc, const int32_t* d_x, int32_t B,
+                                 int32_t n, int32_t* d_terms, int32_t cap, int32_t* d_len, void* cuda_stream) {
+  epic_lexer_table* t = const_cast<epic_lexer_table*>(tc);
+  if (!g || !t || t->g != g || B < 0 || n < 0 || cap < 1) return EPIC_ERR_INVALID_ARG;
+  if (B == 0) return EPIC_OK;
+  if (!d_x || !d_terms || !d_len || n == 0) return EPIC_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  SeqPack sp;
+  epic_status s = region_prepare(g, t, d_x, B, n, sp, st);
+  if (s != EPIC_OK) return s;
+  const size_t per = witness_goal_bytes(cap);
+  s = grow(t, &t->d_wit, &t->wit_bytes, per * (size_t)B);
+  if (s != EPIC_OK) return s;
+  launch_witness(B, st, t->dgl, sp, d_terms, cap, d_len, t->d_wit, t->d_stats);
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
 }
 
@@ -913,6 +1068,10 @@ epic_status epic_get_stats(const epic_lexer_table* t, epic_stats* out, size_t ou
   out->cover_checks = h[S_COVER];
   out->exact_checks = h[S_EXACT];
   out->selected = h[S_SELECTED];
+  out->lex_lookups = h[S_LEX_LOOKUPS];
+  out->lex_misses = h[S_LEX_MISSES];
+  out->lex_uncached = h[S_LEX_UNCACHED];
+  out->witness_failures = h[S_WITNESS_FAIL];
   out->fallback_checks = h[S_FB_CHECKS];
   out->fallback_commits = h[S_FB_COMMITS];
   out->region_checks = t->n_region;

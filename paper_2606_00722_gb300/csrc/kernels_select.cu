@@ -280,7 +280,10 @@ __global__ void __launch_bounds__(kThreads) k_select(DevGrammar g, const LexEntr
 // position that was not rejected and whose update passes the exact test
 // (a whole-graph walk of x (+) c with the Gauss-Seidel columns); a candidate
 // that fails is rejected for good (x only gains commits, and completability
-// is monotone).  Commits go straight into x.  Bounded by the k K candidates.
+// is monotone).  With the single-candidate bits of x before the commits
+// (valid, may be null), a candidate whose bit is 0 is rejected without a
+// walk: its test would fail (monotonicity again).  Commits go straight into
+// x.  Bounded by the k K candidates.
 __global__ void __launch_bounds__(kThreads) k_fallback(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
                                                        int32_t* __restrict__ x, int B, int n,
                                                        const int32_t* __restrict__ pos, int k,
@@ -288,6 +291,7 @@ __global__ void __launch_bounds__(kThreads) k_fallback(DevGrammar g, const LexEn
                                                        const float* __restrict__ conf, int K,
                                                        const int32_t* __restrict__ n_target,
                                                        const uint8_t* __restrict__ selected,
+                                                       const uint8_t* __restrict__ valid,
                                                        int32_t* __restrict__ filled, WsPack wsp,
                                                        unsigned long long* stats) {
   __shared__ WalkShared sh;
@@ -311,7 +315,7 @@ __global__ void __launch_bounds__(kThreads) k_fallback(DevGrammar g, const LexEn
   for (int b = blockIdx.x; b < B; b += gridDim.x) {
     int32_t* xb = x + (long long)b * n;
     for (int j = threadIdx.x; j < k; j += blockDim.x) filled[(long long)b * k + j] = -1;
-    for (int q = threadIdx.x; q < nc; q += blockDim.x) rej[q] = 0;
+    for (int q = threadIdx.x; q < nc; q += blockDim.x) rej[q] = (valid && valid[(long long)b * nc + q] == 0) ? 1 : 0;
     if (threadIdx.x == 0) {
       int nsel = 0;
       if (selected)
@@ -442,12 +446,12 @@ void launch_select(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEnt
 
 void launch_fallback(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab, int32_t* x,
                      int B, int n, const int32_t* pos, int k, const int32_t* cand, const float* conf, int K,
-                     const int32_t* n_target, const uint8_t* selected, int32_t* filled, const WsPack& wsp,
-                     unsigned long long* stats) {
+                     const int32_t* n_target, const uint8_t* selected, const uint8_t* valid, int32_t* filled,
+                     const WsPack& wsp, unsigned long long* stats) {
   const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps);
   cudaFuncSetAttribute(k_fallback, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-  k_fallback<<<grid, kThreads, dyn, st>>>(g, table, vocab, x, B, n, pos, k, cand, conf, K, n_target, selected, filled,
-                                          wsp, stats);
+  k_fallback<<<grid, kThreads, dyn, st>>>(g, table, vocab, x, B, n, pos, k, cand, conf, K, n_target, selected, valid,
+                                          filled, wsp, stats);
 }
 
 }  // namespace epic

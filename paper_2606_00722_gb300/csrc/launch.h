@@ -47,8 +47,13 @@ void launch_select(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEnt
 // Alg. 1's sequential rejection fallback
 void launch_fallback(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab, int32_t* x,
                      int B, int n, const int32_t* pos, int k, const int32_t* cand, const float* conf, int K,
-                     const int32_t* n_target, const uint8_t* selected, int32_t* filled, const WsPack& wsp,
-                     unsigned long long* stats);
+                     const int32_t* n_target, const uint8_t* selected, const uint8_t* valid, int32_t* filled,
+                     const WsPack& wsp, unsigned long long* stats);
+
+// witness extraction (Sec. 4.4) from the forward charts of checks by region
+void launch_witness(int B, cudaStream_t st, const DevGrammar& g, const SeqPack& sp, int32_t* terms, int cap,
+                    int32_t* out_len, void* scratch, unsigned long long* stats);
+size_t witness_goal_bytes(int cap);  // goal and stack scratch per sequence
 
 // measurement builds (EPIC_PHASE_TIMERS): the walk's phase counters of one
 // translation unit, added into out16 (reset: zeroed afterwards)

@@ -52,7 +52,7 @@ inline size_t ws_bytes_per_cta(const WsDims& d, int W, int VW, int FW) {
 
 enum StatIdx {
   S_CHECKS, S_VALID, S_OVERFLOW, S_BAD, S_COLUMNS, S_ENTRIES, S_COVER, S_EXACT, S_SELECTED,
-  S_FB_CHECKS, S_FB_COMMITS, S_N
+  S_FB_CHECKS, S_FB_COMMITS, S_LEX_LOOKUPS, S_LEX_MISSES, S_LEX_UNCACHED, S_WITNESS_FAIL, S_N
 };
 constexpr int kMaxFallbackCand = 4096;  // proposed (position, candidate) pairs per sequence of the fallback
 

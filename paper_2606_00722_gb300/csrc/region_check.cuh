@@ -135,7 +135,13 @@ struct RegionCheck {
       }
     }
     if (nact == 0) return 0;  // nothing of the region passes the node after it (a gap)
+#ifdef EPIC_PHASE_TIMERS
+    long long t_suffix = clock64();
+#endif
     for (int j = rf + 1; j < NF; ++j) {
+#ifdef EPIC_PHASE_TIMERS
+      if (lane == 0) atomicAdd(&g_phase[12], 1ull);  // suffix columns walked
+#endif
       int c = w.open_column();
       if (c < 0) return -1;
       w.res_node = j;
@@ -200,6 +206,12 @@ struct RegionCheck {
       // earlier node can still complete past it, nothing of the region comes back
       if (!keep && a.rec.col_gap[j] && nact == 0) break;
     }
+#ifdef EPIC_PHASE_TIMERS
+    if (lane == 0) {
+      atomicAdd(&g_phase[13], (unsigned long long)(clock64() - t_suffix));
+      atomicAdd(&g_phase[14], 1ull);  // checks that reached the suffix walk
+    }
+#endif
     return w.found ? 1 : 0;
   }
 };

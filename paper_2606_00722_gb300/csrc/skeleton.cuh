@@ -88,16 +88,16 @@ struct Walk {
   // carries all their first terminals.  Returns false on overflow.
   __device__ bool span_step(int tok) {
     int nf = sh.nf;
-    const LexEntry* row = table + (size_t)tok * g.Q;
+    if (g.lazy.stats && threadIdx.x == 0) atomicAdd(&g.lazy.stats[0], (unsigned long long)nf);
     for (int f = threadIdx.x; f < nf; f += blockDim.x) {
-      LexEntry e = row[sc.f_q[f]];
+      LexEntry e = lex_at(g, table, tok, sc.f_q[f]);
       int src = sc.f_c[f];
       int leader = -1;
       if (e.end != 0xFFFF) {
         leader = f;
         for (int h = 0; h < f; ++h) {
           if (sc.f_c[h] != src) continue;
-          LexEntry e2 = row[sc.f_q[h]];
+          LexEntry e2 = lex_at(g, table, tok, sc.f_q[h]);
           if (e2.end != e.end || e2.len != e.len) continue;
           bool same = true;
           for (int t = 1; t < e.len; ++t) same &= e.term[t] == e2.term[t];
@@ -114,7 +114,7 @@ struct Walk {
       int ng = 0;
       for (int f = 0; f < nf; ++f) {
         if (sc.key_q[f] != f) continue;
-        LexEntry e = row[sc.f_q[f]];
+        LexEntry e = lex_at(g, table, tok, sc.f_q[f]);
         sc.g_src[ng] = sc.f_c[f];
         sc.g_end[ng] = e.end;
         sc.g_len[ng] = e.len;
@@ -127,7 +127,7 @@ struct Walk {
         int k = sc.key_q[f];
         if (k == -1) continue;
         int gid = (k <= -2) ? (-2 - k) : (-2 - sc.key_q[k]);
-        LexEntry e = row[sc.f_q[f]];
+        LexEntry e = lex_at(g, table, tok, sc.f_q[f]);
         if (e.len > 0) sc.g_lbl[gid * 8 + (e.term[0] >> 5)] |= 1u << (e.term[0] & 31);
       }
       sh.ng = ng;

@@ -907,7 +907,7 @@ class WarpWalker {
   }
 
   __device__ bool span_step(int tok) {
-    const LexEntry* row = table + (size_t)tok * g.Q;
+    if (g.lazy.stats && wl_lane() == 0) atomicAdd(&g.lazy.stats[0], (unsigned long long)nf);
     int ng = 0;
     PH_BEGIN(t_group);
     // grouping, 32 frontier elements at a time
@@ -917,7 +917,7 @@ class WarpWalker {
       LexEntry e;
       int src = -1;
       if (f < nf) {
-        e = row[ws.f_q[f]];
+        e = lex_at(g, table, tok, ws.f_q[f]);
         src = ws.f_c[f];
         live = e.end != 0xFFFF;
       }

@@ -18,7 +18,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 # translation units, compiled in parallel and linked into one library
 _SRC = [os.path.join(_HERE, 'csrc', f) for f in
         ('epic.cu', 'kernels_walk.cu', 'kernels_select.cu', 'region_forward.cu', 'region_good.cu',
-         'region_check_sm.cu', 'region_check_global.cu', 'peak.cu', 'grammar.cpp')]
+         'region_check_sm.cu', 'region_check_global.cu', 'peak.cu', 'witness.cu', 'grammar.cpp')]
 _DEPS = _SRC + [os.path.join(_HERE, 'csrc', f) for f in
                 ('grammar.h', 'device.cuh', 'walk.cuh', 'cover.cuh', 'skeleton.cuh', 'warpwalk.cuh', 'packs.cuh',
                  'seqpack.cuh', 'launch.h', 'region.cuh', 'region_check.cuh', 'gscols.cuh')] + \
@@ -73,7 +73,8 @@ class _Stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in ('checks', 'valid', 'overflow', 'bad_inputs', 'columns',
                                           'entries', 'cover_checks', 'exact_checks', 'selected',
                                           'region_checks', 'validate_kernels', 'fallback_checks',
-                                          'fallback_commits')]
+                                          'fallback_commits', 'lex_lookups', 'lex_misses', 'lex_uncached',
+                                          'witness_failures')]
 
 
 class _Desc(C.Structure):
@@ -85,9 +86,11 @@ class _Desc(C.Structure):
 
 _lib = None
 EXPORTS = ('epic_grammar_create', 'epic_grammar_destroy', 'epic_grammar_lexer_states',
-           'epic_lexer_table_build', 'epic_lexer_table_destroy', 'epic_lexer_table_copy',
+           'epic_lexer_table_build', 'epic_lexer_table_build_lazy', 'epic_lexer_table_destroy',
+           'epic_lexer_table_copy',
            'epic_validate_batch', 'epic_validate_batch_noalloc',
            'epic_pick_candidates', 'epic_select_compatible_subset', 'epic_commit', 'epic_fallback_commit',
+           'epic_extract_witness',
            'epic_get_stats', 'epic_status_string', 'epic_measure_int_peak', 'epic_last_kernel_times')
 
 
@@ -105,6 +108,7 @@ def load(path: str | None = None):
     lib.epic_grammar_lexer_states.argtypes = [vp]
     lib.epic_grammar_lexer_states.restype = i32
     lib.epic_lexer_table_build.argtypes = [vp, i32p, u8p, i32, vp, C.POINTER(vp)]
+    lib.epic_lexer_table_build_lazy.argtypes = [vp, i32p, u8p, i32, C.c_int64, vp, C.POINTER(vp)]
     lib.epic_lexer_table_destroy.argtypes = [vp]
     lib.epic_lexer_table_copy.argtypes = [vp, i32, i32, vp, C.c_size_t]
     lib.epic_validate_batch.argtypes = [vp, vp, vp, i32, i32, vp, i32, vp, i32, vp, vp]
@@ -112,7 +116,8 @@ def load(path: str | None = None):
     lib.epic_pick_candidates.argtypes = [vp, vp, vp, i32, i32, i32, vp, vp, vp]
     lib.epic_select_compatible_subset.argtypes = [vp, vp, vp, i32, i32, vp, i32, vp, vp, vp, vp]
     lib.epic_commit.argtypes = [vp, i32, i32, vp, i32, vp, vp, vp]
-    lib.epic_fallback_commit.argtypes = [vp, vp, vp, i32, i32, vp, i32, vp, vp, i32, vp, vp, vp, vp]
+    lib.epic_fallback_commit.argtypes = [vp, vp, vp, i32, i32, vp, i32, vp, vp, i32, vp, vp, vp, vp, vp]
+    lib.epic_extract_witness.argtypes = [vp, vp, vp, i32, i32, vp, i32, vp, vp]
     lib.epic_get_stats.argtypes = [vp, C.POINTER(_Stats), C.c_size_t, C.c_int]
     lib.epic_measure_int_peak.argtypes = [C.POINTER(C.c_double), C.POINTER(C.c_double), vp]
     lib.epic_measure_int_peak.restype = C.c_int
@@ -194,16 +199,24 @@ class Grammar:
 class LexTable:
     """epic_lexer_table_build / epic_lexer_table_destroy."""
 
-    def __init__(self, grammar: Grammar, vocab, stream=None):
+    def __init__(self, grammar: Grammar, vocab, stream=None, lazy_capacity: int | None = None):
+        """lazy_capacity: build lazily (epic_lexer_table_build_lazy) with a
+        memo of that many entries, instead of the dense table."""
         lib = load()
         lens = np.array([len(t) for t in vocab], np.int64)
         off = np.zeros(len(vocab) + 1, np.int32)
         off[1:] = np.cumsum(lens)
         data = np.frombuffer(b''.join(vocab), np.uint8).copy()
         h = C.c_void_p()
-        _check(lib.epic_lexer_table_build(grammar.h, off.ctypes.data_as(C.POINTER(C.c_int32)),
-                                          data.ctypes.data_as(C.POINTER(C.c_uint8)), len(vocab),
-                                          _stream(stream), C.byref(h)), 'epic_lexer_table_build')
+        if lazy_capacity is None:
+            _check(lib.epic_lexer_table_build(grammar.h, off.ctypes.data_as(C.POINTER(C.c_int32)),
+                                              data.ctypes.data_as(C.POINTER(C.c_uint8)), len(vocab),
+                                              _stream(stream), C.byref(h)), 'epic_lexer_table_build')
+        else:
+            _check(lib.epic_lexer_table_build_lazy(grammar.h, off.ctypes.data_as(C.POINTER(C.c_int32)),
+                                                   data.ctypes.data_as(C.POINTER(C.c_uint8)), len(vocab),
+                                                   int(lazy_capacity), _stream(stream), C.byref(h)),
+                   'epic_lexer_table_build_lazy')
         self.h = h
         self.grammar = grammar
         self.vocab = len(vocab)
@@ -299,15 +312,17 @@ def commit(x, pos, tok, selected, stream=None):
            'epic_commit')
 
 
-def fallback_commit(g: Grammar, t: LexTable, x, pos, cand, cand_conf, n_target, selected, filled, stream=None):
+def fallback_commit(g: Grammar, t: LexTable, x, pos, cand, cand_conf, n_target, selected, filled, stream=None,
+                    valid=None):
     """epic_fallback_commit: Alg. 1's sequential rejection fallback (selected
-    may be None for an empty batch B)."""
+    may be None for an empty batch B; valid, the single-candidate bits of x
+    before the commits, lets it skip candidates that would fail)."""
     B, n = x.shape
     k = pos.shape[1]
     K = cand.shape[2]
     _check(load().epic_fallback_commit(g.h, t.h, _ptr(x), B, n, _ptr(pos), k, _ptr(cand), _ptr(cand_conf), K,
-                                       _ptr(n_target), _ptr(selected), _ptr(filled), _stream(stream)),
-           'epic_fallback_commit')
+                                       _ptr(n_target), _ptr(selected), _ptr(valid), _ptr(filled),
+                                       _stream(stream)), 'epic_fallback_commit')
 
 
 def decode_step(g: Grammar, t: LexTable, x, pos, cand, cand_conf, n_target, bufs, stream=None):
@@ -321,4 +336,16 @@ def decode_step(g: Grammar, t: LexTable, x, pos, cand, cand_conf, n_target, bufs
     pick_candidates(cand, cand_conf, bufs['valid'], bufs['tok'], bufs['conf'], stream)
     select_compatible_subset(g, t, x, pos, bufs['tok'], bufs['conf'], bufs['selected'], stream)
     commit(x, pos, bufs['tok'], bufs['selected'], stream)
-    fallback_commit(g, t, x, pos, cand, cand_conf, n_target, bufs['selected'], bufs['filled'], stream)
+    fallback_commit(g, t, x, pos, cand, cand_conf, n_target, bufs['selected'], bufs['filled'], stream,
+                    valid=bufs['valid'])
+
+
+GAP_BIT = 1 << 16  # a witness terminal produced inside a mask run
+
+
+def extract_witness(g: Grammar, t: LexTable, x, terms, lengths, stream=None):
+    """epic_extract_witness: terms [B][cap] int32 (terminal | GAP_BIT when a
+    gap produces it), lengths [B] int32 (-1: not completable, -2: capacity)."""
+    B, n = x.shape
+    _check(load().epic_extract_witness(g.h, t.h, _ptr(x), B, n, _ptr(terms), terms.shape[1], _ptr(lengths),
+                                       _stream(stream)), 'epic_extract_witness')

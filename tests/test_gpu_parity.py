@@ -144,5 +144,62 @@ def test_decode_step_with_fallback(cuda, name, seed, kw, fill):
     np.testing.assert_array_equal(bufs['selected'].cpu().numpy(), ref_sel)
     np.testing.assert_array_equal(bufs['filled'].cpu().numpy(), ref_filled)
     np.testing.assert_array_equal(x.cpu().numpy(), ref_x)
-    assert st['fallback_checks'] == nchk
+    # decode_step hands the fallback the step's validity bits, so it tests
+    # only candidates whose bit is not 0 (the others would fail their test)
+    assert st['fallback_checks'] <= nchk
     assert st['fallback_commits'] == int((ref_filled >= 0).sum())
+    # without the bits every candidate is tested, as in the oracle's loop
+    x2 = _dev(x1, cuda)
+    filled2 = torch.empty(w.pos.shape, dtype=torch.int32, device=cuda)
+    t.stats(reset=True)
+    epic.fallback_commit(g, t, x2, _dev(w.pos, cuda), _dev(w.cand, cuda), _dev(w.conf, cuda), _dev(n_target, cuda),
+                         _dev(ref_sel, cuda), filled2)
+    torch.cuda.synchronize()
+    st2 = t.stats()
+    np.testing.assert_array_equal(filled2.cpu().numpy(), ref_filled)
+    np.testing.assert_array_equal(x2.cpu().numpy(), ref_x)
+    assert st2['fallback_checks'] == nchk
+
+
+def _step_with_table(w, dev, lazy_capacity):
+    import torch
+    import paper_2606_00722_gb300 as epic
+    g = epic.Grammar(w.grammar)
+    t = epic.LexTable(g, w.vocab, lazy_capacity=lazy_capacity)
+    x = _dev(w.x, dev)
+    pos = _dev(w.pos, dev)
+    cand = _dev(w.cand, dev)
+    conf3 = _dev(w.conf, dev)
+    bufs = dict(valid=torch.empty(w.cand.shape, dtype=torch.uint8, device=dev),
+                tok=torch.empty(w.pos.shape, dtype=torch.int32, device=dev),
+                conf=torch.empty(w.pos.shape, dtype=torch.float32, device=dev),
+                selected=torch.empty(w.pos.shape, dtype=torch.uint8, device=dev),
+                filled=torch.empty(w.pos.shape, dtype=torch.int32, device=dev))
+    epic.decode_step(g, t, x, pos, cand, conf3, _dev(np.full(w.B, w.k, np.int32), dev), bufs)
+    torch.cuda.synchronize()
+    return {k: v.cpu().numpy() for k, v in bufs.items()}, x.cpu().numpy(), t.stats()
+
+
+@pytest.mark.parametrize('name,seed,kw', [
+    ('expr-tiny', 42, {}), ('json-schema', 42, dict(batch=4)), ('smiles-256', 43, dict(batch=6, k=4)),
+    ('clike-512', 42, dict(batch=1, k=2, K=4, n=128)),
+])
+def test_lazy_lex_memo_equals_dense_table(cuda, name, seed, kw):
+    """Alg. 2's lexing memo filled on first use (no dense table): whole steps
+    identical to those with the dense table, with a memo large enough to hold
+    every entry used and with one too small for most (entries then computed
+    without being stored); the counters give the memo's hit rate."""
+    w = make_workload(name, seed, **kw)
+    ref, ref_x, ref_st = _step_with_table(w, cuda, None)
+    assert ref_st['lex_lookups'] > 0 and ref_st['lex_misses'] == 0
+    for cap in (1 << 20, 64):
+        got, got_x, st = _step_with_table(w, cuda, cap)
+        for key in ('valid', 'selected', 'filled'):
+            np.testing.assert_array_equal(got[key], ref[key])
+        np.testing.assert_array_equal(got_x, ref_x)
+        assert st['lex_lookups'] == ref_st['lex_lookups']
+        assert 0 < st['lex_misses'] <= st['lex_lookups']
+        if cap == 64:
+            assert st['lex_uncached'] > 0
+        else:
+            assert st['lex_uncached'] == 0 and st['lex_misses'] < st['lex_lookups']

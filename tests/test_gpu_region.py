@@ -138,3 +138,23 @@ def test_random_stress_full_length_row(cuda):
     assert st['overflow'] == 0
     assert st['region_checks'] == cand.size
     np.testing.assert_array_equal(got[0], np.array(gold['valid'], np.uint8))
+
+
+def test_clike_full_batch_sampled(cuda):
+    """The clike-512 benchmark batch (32 x 512, k = 8, K = 32) in one
+    epic_validate_batch call, the launch bench.py times, against the oracle's
+    bits for a sample of 128 of its checks (every candidate of four
+    (sequence, position) pairs), stored by tests/golden/make_sample_golden.py
+    (the whole batch is about 8,000 oracle checks of 512-token rows)."""
+    import json
+    here = os.path.dirname(os.path.abspath(__file__))
+    with open(os.path.join(here, 'golden', 'sample_clike-512.json')) as f:
+        gold = json.load(f)
+    w = make_workload(gold['workload'], gold['seed'])
+    assert (w.B, w.x.shape[1], w.k, w.K) == (gold['batch'], gold['n'], gold['k'], gold['K'])
+    got, st = run_gpu(w.grammar, w.vocab, w.x, w.pos, w.cand, cuda)
+    assert st['overflow'] == 0
+    assert st['checks'] == w.cand.size
+    for c in gold['checks']:
+        assert got[c['b'], c['j'], c['c']] == c['valid'], c
+    assert any(c['valid'] for c in gold['checks']) and not all(c['valid'] for c in gold['checks'])
