@@ -116,7 +116,8 @@ epic_status epic_lexer_table_build(const epic_grammar* g, const int32_t* tok_off
  * two, at most 2^30) keyed by (token, lexer state) is filled by the walks,
  * each entry computed by the transducer above on its first lookup.  Every
  * call gives the same results as with the dense table.  A lookup that finds
- * no free slot within 64 probes computes its entry without storing it
+ * no free slot within 64 probes, or finds its entry still being computed by
+ * another thread after a bounded wait, computes the entry without storing it
  * (stats.lex_uncached).  Counters: stats.lex_lookups, stats.lex_misses (the
  * memo's hit rate is 1 - misses / lookups).  Errors as epic_lexer_table_build,
  * plus EPIC_ERR_CAPACITY when vocab x states does not fit 32-bit keys.
@@ -259,13 +260,18 @@ epic_status epic_commit(int32_t* d_x, int32_t B, int32_t n, const int32_t* d_pos
  * whose bit is 0 is rejected without a test (it would fail it: a partial
  * output that is not completable stays so after more commits, App. D); the
  * result is the same with or without it.  Output d_filled [B][k] int32: the
- * token this call committed at slot j, else -1.  One CTA per sequence; each
- * test is a whole-graph walk of x (+) c.
+ * token this call committed at slot j, else -1.  Each test is a whole-graph
+ * walk of x (+) c by one CTA.  The loop runs in rounds: up to 16 CTAs per
+ * sequence test its next candidates in order against the same x at once,
+ * and the round is then read in that order (failures reject, the first pass
+ * commits; after it, failures still reject and passes are tested again), so
+ * the commits are the sequential loop's.
  * Errors: EPIC_ERR_INVALID_ARG (NULL pointers, sizes < 0),
  * EPIC_ERR_CAPACITY when k K > 4096.  A NaN confidence or a position out of
  * range leaves that sequence unchanged (stats.bad_inputs); a test that hits
- * a capacity limit ends that sequence's loop (stats.overflow).
- * Asynchronous.
+ * a capacity limit rejects its candidate (stats.overflow).
+ * Synchronizes with the stream once per round (it reads whether any
+ * sequence still wants commits); stats.fallback_rounds counts the rounds.
  */
 epic_status epic_fallback_commit(const epic_grammar* g, const epic_lexer_table* t, int32_t* d_x, int32_t B,
                                  int32_t n, const int32_t* d_pos, int32_t k, const int32_t* d_cand,
@@ -309,8 +315,9 @@ typedef struct {
   uint64_t fallback_commits; /* candidates it committed                       */
   uint64_t lex_lookups;      /* (token, lexer state) lookups of span lexing   */
   uint64_t lex_misses;       /* lazy tables: entries computed on first use    */
-  uint64_t lex_uncached;     /* lazy tables: computed without a free slot     */
+  uint64_t lex_uncached;     /* lazy tables: computed without being stored    */
   uint64_t witness_failures; /* witness searches that found no derivation     */
+  uint64_t fallback_rounds;  /* rounds of epic_fallback_commit (2 launches each) */
 } epic_stats;
 
 /* Copy the counters (synchronizes the lexer table's last stream); out_bytes

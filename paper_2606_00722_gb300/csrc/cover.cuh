@@ -75,14 +75,15 @@ class CoverCols {
     for (int w = threadIdx.x; w < FW; w += blockDim.x) R[w] = 0;
     __syncthreads();
     int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // each warp takes every kWarps-th set state and ORs its closure row
+    const int nwarps = blockDim.x >> 5;
+    // each warp takes every nwarps-th set state and ORs its closure row
     int seen = 0;
     for (int w = 0; w < FW; ++w) {
       uint32_t m = S[w];
       while (m) {
         int b = __ffs(m) - 1;
         m &= m - 1;
-        if ((seen++ % kWarps) != warp) continue;
+        if ((seen++ % nwarps) != warp) continue;
         const uint32_t* r = rows + (size_t)((w << 5) + b) * FW;
         for (int v = lane; v < FW; v += 32)
           if (r[v]) atomicOr(&R[v], r[v]);

@@ -66,6 +66,7 @@ struct DevGrammar {
   const int32_t* nt_comp;
   const int32_t* ny_off;          // [V+1]
   const int32_t* ny;
+  int gs_par;                     // CTA walks: warp-parallel origin sweep (gscols.cuh)
 };
 
 // The greedy transducer of one token from lexer state q (Sec. 4.1): at state
@@ -135,7 +136,9 @@ __device__ inline LexEntry lex_at(const DevGrammar& g, const LexEntry* table, in
       }
     }
     if (k == key) {
-      for (int spin = 0; spin < (1 << 16); ++spin)
+      // published by its owner, possibly a lane of this warp on another
+      // branch: sleep between polls so that it runs
+      for (int spin = 0; spin < (1 << 16); ++spin, __nanosleep(32))
         if (*((volatile const uint32_t*)&L.ready[h])) {
           __threadfence();
           const volatile uint32_t* v = reinterpret_cast<const volatile uint32_t*>(&L.vals[h]);

@@ -102,6 +102,9 @@ struct epic_lexer_table {
   int32_t* d_regs = nullptr; // per-warp tables of region checks
   char* d_wit = nullptr;     // witness extraction: goals and stack per sequence
   size_t wit_bytes = 0;
+  char* d_fb = nullptr;      // rejection fallback: rejections, state and round results per sequence
+  size_t fb_bytes = 0;
+  mutable unsigned long long n_fb_rounds = 0;  // host-side counter: fallback rounds launched
   size_t regs_bytes = 0;
   int spec_cap = 0;
   char* d_wws = nullptr;   // warp-walk workspace
@@ -773,6 +776,7 @@ void epic_lexer_table_destroy(epic_lexer_table* t) {
   cudaFree(t->d_seq);
   cudaFree(t->d_regs);
   cudaFree(t->d_wit);
+  cudaFree(t->d_fb);
   cudaFree(t->d_stats);
   cudaFree(t->d_counter);
   cudaFree(t->d_lz_keys);
@@ -1018,11 +1022,41 @@ epic_status epic_fallback_commit(const epic_grammar* g, const epic_lexer_table* 
   if (!d_x || !d_pos || !d_cand || !d_cand_conf || !d_n_target || !d_filled || n == 0 || K == 0)
     return EPIC_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)cuda_stream;
-  epic_status s = ensure_workspace(t, std::min(B, sm_count() * 2), n, st);
+  const int nc = k * K;
+  // rounds of m tests per sequence, as many CTAs as two per SM (at most
+  // kMaxFallbackSpec tests per sequence, at least one)
+  int m = std::max(1, std::min(kMaxFallbackSpec, std::min(nc, (2 * sm_count()) / B)));
+  epic_status s = ensure_workspace(t, std::min((long long)B * m, (long long)sm_count() * 2), n, st);
+  if (s != EPIC_OK) return s;
+  m = std::max(1, std::min(m, t->ctas / B));
+  auto r16 = [](size_t b) { return (b + 15) & ~(size_t)15; };
+  const size_t o_fb = r16((size_t)B * nc), o_res = o_fb + r16((size_t)B * 2 * 4),
+               o_act = o_res + r16((size_t)B * m * 2 * 4), need = o_act + 16;
+  s = grow(t, &t->d_fb, &t->fb_bytes, need);
   if (s != EPIC_OK) return s;
   t->last = st;
-  launch_fallback(std::min(B, t->ctas), st, t->dgl, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_cand, d_cand_conf, K,
-                  d_n_target, d_selected, d_valid, d_filled, pack_of(t), t->d_stats);
+  uint8_t* rej = (uint8_t*)t->d_fb;
+  int32_t* fb = (int32_t*)(t->d_fb + o_fb);
+  int32_t* res = (int32_t*)(t->d_fb + o_res);
+  unsigned long long* act = (unsigned long long*)(t->d_fb + o_act);
+  unsigned long long h_act = 0;
+  auto read_active = [&]() -> bool {
+    if (cudaMemcpyAsync(&h_act, act, 8, cudaMemcpyDeviceToHost, st) != cudaSuccess) return false;
+    return cudaStreamSynchronize(st) == cudaSuccess;
+  };
+  if (cudaMemsetAsync(act, 0, 8, st) != cudaSuccess) return EPIC_ERR_CUDA;
+  launch_fallback_init(B, st, n, d_pos, k, d_cand_conf, K, d_n_target, d_selected, d_valid, d_filled, rej, fb, act,
+                       t->d_stats);
+  if (!read_active()) return EPIC_ERR_CUDA;
+  const int grid = (int)std::min<long long>((long long)B * m, t->ctas);
+  for (int round = 0; round <= nc && h_act > 0; ++round) {  // each round rejects or commits a candidate
+    launch_fallback_round(grid, st, t->dgl, t->d_table, t->vocab, d_x, B, n, d_pos, k, d_cand, d_cand_conf, K, m, rej,
+                          fb, res, pack_of(t), t->d_stats);
+    if (cudaMemsetAsync(act, 0, 8, st) != cudaSuccess) return EPIC_ERR_CUDA;
+    launch_fallback_resolve(B, st, d_x, n, d_pos, k, d_cand, K, m, rej, fb, res, d_filled, act, t->d_stats);
+    ++t->n_fb_rounds;
+    if (!read_active()) return EPIC_ERR_CUDA;
+  }
   return cudaGetLastError() == cudaSuccess ? EPIC_OK : EPIC_ERR_CUDA;
 }
 
@@ -1072,6 +1106,7 @@ epic_status epic_get_stats(const epic_lexer_table* t, epic_stats* out, size_t ou
   out->lex_misses = h[S_LEX_MISSES];
   out->lex_uncached = h[S_LEX_UNCACHED];
   out->witness_failures = h[S_WITNESS_FAIL];
+  out->fallback_rounds = t->n_fb_rounds;
   out->fallback_checks = h[S_FB_CHECKS];
   out->fallback_commits = h[S_FB_COMMITS];
   out->region_checks = t->n_region;
@@ -1080,6 +1115,7 @@ epic_status epic_get_stats(const epic_lexer_table* t, epic_stats* out, size_t ou
     if (cudaMemset(t->d_stats, 0, sizeof(h)) != cudaSuccess) return EPIC_ERR_CUDA;
     t->n_region = 0;
     t->n_vkernels = 0;
+    t->n_fb_rounds = 0;
   }
   return EPIC_OK;
 }

@@ -27,6 +27,23 @@ namespace epic {
 
 constexpr int kGsMaxWarps = 16;
 constexpr long long kGsMaxSteps = 1ll << 22;  // origin visits per column
+constexpr long long kGsMaxIdle = 1ll << 24;   // polls of an idle warp per column (warp-parallel sweep)
+
+// Per-warp scratch of the warp-parallel sweep (dynamic shared memory):
+// nonterminal words, then the warp's completion mask.
+constexpr int kGsWarpScratch = kMaxVW + kMaxW;
+__host__ __device__ inline size_t gs_warp_scratch_bytes() { return (size_t)kGsMaxWarps * kGsWarpScratch * 4; }
+
+// The origin sweep of the CTA walks: warp-parallel for item sets of at most
+// 64 words, whose columns are short enough for one warp to scatter (on
+// clike-512, W = 64: forward charts 22 % faster), the descending block sweep
+// for wider ones (random-stress-1024, W = 213: the warp-parallel sweep took
+// 20-45 % longer, one warp scattering columns of hundreds of entries);
+// EPIC_GS_PARALLEL=0/1 overrides.
+inline int gs_parallel_enabled(int W) {
+  const char* e = getenv("EPIC_GS_PARALLEL");
+  return e ? (atoi(e) != 0) : (W <= 64 ? 1 : 0);
+}
 
 // Shared memory of the Gauss-Seidel columns (beside WalkShared).
 struct GsShared {
@@ -39,6 +56,7 @@ struct GsShared {
   int32_t cur_o;
   int32_t flag;
   int32_t labelled;  // the open column has a labelled arrival (else only epsilon ones)
+  int32_t busy;      // warp-parallel sweep: warps holding an origin
 };
 
 // Grammar tables read by the per-item loops, staged in shared memory:
@@ -97,6 +115,11 @@ class EarleyColsGS {
   static constexpr bool kRecord = REC;
   const BlockRec* rec = nullptr;
   uint32_t* wnt = nullptr;  // recording walks: per-warp nonterminal sets [warps][kMaxVW] (shared memory)
+  // Warp-parallel sweep (set both): every warp claims dirty origins on its
+  // own and scatters their completions alone; ws.bdone keeps, per origin of
+  // the open column, the nonterminals whose completions were scattered.
+  bool par = false;
+  uint32_t* wscr = nullptr;  // [warps][kGsWarpScratch] (shared memory)
 
   __device__ EarleyColsGS(const DevGrammar& g_, const GsTables& t_, const LexEntry* t, Workspace w, WalkScratch s,
                           WsDims d, WalkShared& shared, GsShared& gss)
@@ -466,6 +489,282 @@ class EarleyColsGS {
     __syncthreads();
   }
 
+  // ------------------------------------------------------ warp-parallel sweep
+  // The same least fixpoint as the descending sweep, reached without block
+  // barriers: each warp repeatedly claims the highest dirty origin below c
+  // (clearing its bit), closes its row with the self-loop, claims in
+  // ws.bdone the nonterminals it completes that no visit scattered yet, and
+  // scatters those over column o with atomic ORs, marking the rows it changes
+  // dirty again.  A row may be claimed while another warp still writes into
+  // it; the writer sets the dirty bit after its writes (fenced), so the row
+  // is visited again and nothing is lost.  The sweep ends when no bit is
+  // dirty and no warp holds an origin.  Rows are read through L2 (ld.cg):
+  // other warps' atomics do not update this SM's L1.
+
+  __device__ static int warp_highest_dirty(const uint32_t* bm, int top) {
+    const int lane = threadIdx.x & 31;
+    if (top < 0) return -1;
+    const volatile uint32_t* vb = bm;
+    for (int wtop = top >> 5; wtop >= 0; wtop -= 32) {
+      const int w = wtop - lane;
+      uint32_t v = (w >= 0) ? vb[w] : 0u;
+      if (w == (top >> 5)) v &= (top & 31) == 31 ? 0xffffffffu : ((2u << (top & 31)) - 1u);
+      const unsigned any = __ballot_sync(0xffffffffu, v != 0);
+      if (any) {
+        const int l = __ffs(any) - 1;
+        const uint32_t vv = __shfl_sync(0xffffffffu, v, l);
+        return ((wtop - l) << 5) + (31 - __clz(vv));
+      }
+    }
+    return -1;
+  }
+
+  // Warp: close row o with its self-loop (as close_origin), the nonterminals
+  // already scattered for o taken as done; returns, in lane v < VW, word v of
+  // the nonterminals this visit claimed (completed from o and not yet
+  // scattered by any visit).
+  __device__ uint32_t close_origin_claim(int o, int mode, uint32_t* nstep) {
+    const int lane = threadIdx.x & 31;
+    uint32_t* row = ws.stage + (size_t)o * W;
+    uint32_t* bd = ws.bdone + (size_t)o * VW;
+    // done before the row: a visit writes its row before it claims
+    uint32_t known = (lane < VW) ? __ldcg(bd + lane) : 0u;
+    __threadfence_block();
+    uint32_t r[KW], r0[KW], e[KW];
+#pragma unroll
+    for (int i = 0; i < KW; ++i) {
+      const int w = lane + 32 * i;
+      r[i] = (w < W) ? __ldcg(row + w) : 0u;
+      r0[i] = r[i];
+      e[i] = 0u;
+    }
+    const int kb = ws.col_off[o], ke = ws.col_off[o + 1];
+    const bool self = ke > kb && ws.org[ke - 1] == o;
+    if (self) {
+      const uint32_t* E = ws.bits + (size_t)(ke - 1) * W;
+#pragma unroll
+      for (int i = 0; i < KW; ++i) {
+        const int w = lane + 32 * i;
+        e[i] = (w < W) ? (E[w] & tb.any_nt[w]) : 0u;
+      }
+    }
+    uint32_t tot = 0;
+    uint32_t cseen[KW];
+#pragma unroll
+    for (int i = 0; i < KW; ++i) cseen[i] = 0u;
+    for (int round = 0; round < 64 * kMaxW; ++round) {
+      reg_advance(r, mode);
+      if (lane < VW) nstep[lane] = 0;
+      __syncwarp();
+#pragma unroll
+      for (int i = 0; i < KW; ++i) {
+        const int w = lane + 32 * i;
+        uint32_t m = (w < W) ? (r[i] & tb.complete[w] & ~cseen[i]) : 0u;
+        cseen[i] |= m;
+        while (m) {
+          const int b = __ffs(m) - 1;
+          m &= m - 1;
+          const int A = tb.item_lhs[(w << 5) + b];
+          atomicOr(&nstep[A >> 5], 1u << (A & 31));
+        }
+      }
+      __syncwarp();
+      const uint32_t nw = (lane < VW) ? (nstep[lane] & ~known) : 0u;
+      known |= nw;
+      tot |= nw;
+      if (!__any_sync(0xffffffffu, nw != 0) || !self) break;
+      if (lane < VW) nstep[lane] = nw;
+      __syncwarp();
+      bool ch = false;
+      uint32_t carry = 0;
+#pragma unroll
+      for (int i = 0; i < KW; ++i) {
+        if (32 * i >= W) break;
+        const int w = lane + 32 * i;
+        uint32_t x = 0, m = e[i];
+        while (m) {
+          const int b = __ffs(m) - 1;
+          m &= m - 1;
+          const int B = tb.item_next[(w << 5) + b] - g.T;
+          if ((nstep[B >> 5] >> (B & 31)) & 1u) x |= 1u << b;
+        }
+        uint32_t prev = __shfl_up_sync(0xffffffffu, x, 1);
+        if (lane == 0) prev = carry;
+        carry = __shfl_sync(0xffffffffu, x, 31);
+        const uint32_t add = ((x << 1) | (prev >> 31)) & ~r[i];
+        ch |= add != 0;
+        r[i] |= add;
+      }
+      __syncwarp();
+      if (!__any_sync(0xffffffffu, ch)) break;
+    }
+#pragma unroll
+    for (int i = 0; i < KW; ++i) {
+      const int w = lane + 32 * i;
+      if (w < W && (r[i] & ~r0[i])) atomicOr(row + w, r[i]);
+    }
+    __threadfence_block();
+    uint32_t mine = 0;
+    if (lane < VW && tot) mine = tot & ~atomicOr(bd + lane, tot);
+    return mine;
+  }
+
+  // Warp: completions of the nonterminals in nnew (nnew[v], v < VW) from
+  // origin o into the rows of the other entries of column o.
+  __device__ void scatter_warp(int o, const uint32_t* nnew, uint32_t* expn) {
+    const int lane = threadIdx.x & 31;
+    for (int w = lane; w < W; w += 32) {
+      uint32_t acc = 0, m = tb.any_nt[w];
+      while (m) {
+        const int b = __ffs(m) - 1;
+        m &= m - 1;
+        const int B = tb.item_next[(w << 5) + b] - g.T;
+        if ((nnew[B >> 5] >> (B & 31)) & 1u) acc |= 1u << b;
+      }
+      expn[w] = acc;
+    }
+    __syncwarp();
+    uint32_t ex[KW];
+#pragma unroll
+    for (int i = 0; i < KW; ++i) {
+      const int w = lane + 32 * i;
+      ex[i] = (w < W) ? expn[w] : 0u;
+    }
+    const int kb = ws.col_off[o], ke = ws.col_off[o + 1];
+    const bool self = ke > kb && ws.org[ke - 1] == o;
+    const int nsc = (self ? ke - 1 : ke) - kb;
+    const uint32_t* __restrict__ bits = ws.bits + (size_t)kb * W;
+    for (int e0 = 0; e0 < nsc; e0 += 2) {
+      const bool has1 = e0 + 1 < nsc;
+      const uint32_t* s0 = bits + (size_t)e0 * W;
+      const uint32_t* s1 = bits + (size_t)(has1 ? e0 + 1 : e0) * W;
+      uint32_t v0[KW], v1[KW];
+#pragma unroll
+      for (int i = 0; i < KW; ++i) {
+        const int w = lane + 32 * i;
+        v0[i] = ex[i] ? (__ldg(s0 + w) & ex[i]) : 0u;
+        v1[i] = (ex[i] && has1) ? (__ldg(s1 + w) & ex[i]) : 0u;
+      }
+      const int o0 = ws.org[kb + e0], o1 = ws.org[kb + (has1 ? e0 + 1 : e0)];
+      uint32_t* d0 = ws.stage + (size_t)o0 * W;
+      uint32_t* d1 = ws.stage + (size_t)o1 * W;
+      uint32_t a0[KW], a1[KW];
+      {
+        uint32_t c0 = 0, c1 = 0;
+#pragma unroll
+        for (int i = 0; i < KW; ++i) {
+          uint32_t p0 = __shfl_up_sync(0xffffffffu, v0[i], 1);
+          uint32_t p1 = __shfl_up_sync(0xffffffffu, v1[i], 1);
+          if (lane == 0) {
+            p0 = c0;
+            p1 = c1;
+          }
+          c0 = __shfl_sync(0xffffffffu, v0[i], 31);
+          c1 = __shfl_sync(0xffffffffu, v1[i], 31);
+          a0[i] = (v0[i] << 1) | (p0 >> 31);
+          a1[i] = has1 ? ((v1[i] << 1) | (p1 >> 31)) : 0u;
+        }
+      }
+      uint32_t q0[KW], q1[KW];
+#pragma unroll
+      for (int i = 0; i < KW; ++i) {
+        const int w = lane + 32 * i;
+        q0[i] = (w < W && a0[i]) ? __ldcg(d0 + w) : 0u;
+        q1[i] = (w < W && a1[i]) ? __ldcg(d1 + w) : 0u;
+      }
+      bool ch0 = false, ch1 = false;
+#pragma unroll
+      for (int i = 0; i < KW; ++i) {
+        const int w = lane + 32 * i;
+        if (w < W && (a0[i] & ~q0[i])) {
+          atomicOr(d0 + w, a0[i]);
+          ch0 = true;
+        }
+        if (w < W && (a1[i] & ~q1[i])) {
+          atomicOr(d1 + w, a1[i]);
+          ch1 = true;
+        }
+      }
+      __threadfence_block();  // every lane's row writes before the dirty bits
+      ch0 = __any_sync(0xffffffffu, ch0);
+      ch1 = __any_sync(0xffffffffu, ch1);
+      __syncwarp();
+      if (lane == 0) {
+        if (ch0) {
+          atomicOr(&sh.touched[o0 >> 5], 1u << (o0 & 31));
+          atomicOr(&sh.dirty[o0 >> 5], 1u << (o0 & 31));
+        }
+        if (ch1 && has1) {
+          atomicOr(&sh.touched[o1 >> 5], 1u << (o1 & 31));
+          atomicOr(&sh.dirty[o1 >> 5], 1u << (o1 & 31));
+        }
+      }
+      __syncwarp();
+    }
+  }
+
+  // Block: the origins below c, closed warp-parallel (every warp returns
+  // when the sweep is done).
+  __device__ void close_origins_par(int c, int mode) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint32_t* nstep = wscr + (size_t)warp * kGsWarpScratch;
+    uint32_t* expn = nstep + kMaxVW;
+    volatile int32_t* busy = &gs.busy;
+    long long visits = 0, idle = 0;
+    for (;;) {
+      // claim the highest dirty origin; a holder counts itself busy right
+      // after its claim (a warp that saw nothing dirty and no holder in that
+      // gap leaves early, and the holder finishes what its origin causes)
+      int o = -1;
+      for (int tries = 0; tries < 64; ++tries) {
+        const int h = warp_highest_dirty(sh.dirty, c - 1);
+        if (h < 0) break;
+        uint32_t old = 0;
+        if (lane == 0) {
+          old = atomicAnd(&sh.dirty[h >> 5], ~(1u << (h & 31)));
+          if ((old >> (h & 31)) & 1u) atomicAdd(&gs.busy, 1);
+        }
+        old = __shfl_sync(0xffffffffu, old, 0);
+        if ((old >> (h & 31)) & 1u) {
+          o = h;
+          break;
+        }
+      }
+      if (o < 0) {
+        // done when no warp holds an origin and, after that, nothing is dirty
+        int b = 0;
+        if (lane == 0) b = *busy;
+        b = __shfl_sync(0xffffffffu, b, 0);
+        __threadfence_block();
+        if (b == 0 && warp_highest_dirty(sh.dirty, c - 1) < 0) break;
+        if (++idle > kGsMaxIdle) {
+          if (lane == 0) sh.status = kWalkOverflow;
+          break;
+        }
+        __nanosleep(64);
+        continue;
+      }
+      __syncwarp();  // the claim (lane 0) before any lane reads the row
+      __threadfence_block();
+      if (++visits > kGsMaxSteps) {
+        if (lane == 0) {
+          sh.status = kWalkOverflow;
+          atomicSub(&gs.busy, 1);
+        }
+        __syncwarp();
+        break;
+      }
+      const uint32_t mine = close_origin_claim(o, mode, nstep);
+      if (lane < VW) nstep[lane] = mine;
+      __syncwarp();
+      if (__any_sync(0xffffffffu, mine != 0)) scatter_warp(o, nstep, expn);
+      __threadfence_block();
+      __syncwarp();
+      if (lane == 0) atomicSub(&gs.busy, 1);
+      __syncwarp();
+    }
+  }
+
   // Closure of column c (gap: a node with a Sigma_lex* self-loop).
   __device__ void close_column(int c, bool gap) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = nwarps();
@@ -479,6 +778,14 @@ class EarleyColsGS {
     //    an origin completes here, it completed in one of the sources, whose
     //    rows below already hold the advanced items).
     int top = (!gap && !gs.labelled) ? -1 : c - 1;
+    if (par) {
+      if (threadIdx.x == 0) gs.busy = 0;
+      __syncthreads();
+      if (top >= 0) close_origins_par(c, mode);
+      __syncthreads();
+      if (sh.status == kWalkOverflow) return;
+      top = -1;  // the descending sweep below has nothing left
+    }
     for (long long step = 0;; ++step) {
       if (warp == 0) {
         PH_BEGIN(t_or);
@@ -656,6 +963,8 @@ class EarleyColsGS {
       }
       __syncwarp();
       for (int w = lane; w < W; w += 32) row[w] = 0;
+      if (par)
+        for (int v = lane; v < VW; v += 32) ws.bdone[(size_t)o * VW + v] = 0;
     }
     clear_bitmap(sh.touched, c + 1);
     clear_bitmap(sh.dirty, c + 1);
@@ -719,6 +1028,8 @@ class EarleyColsGS {
     for (int i = warp; i < nl; i += nw) {
       const int o = sh.list[i];
       for (int w = lane; w < W; w += 32) ws.stage[(size_t)o * W + w] = 0;
+      if (par)
+        for (int v = lane; v < VW; v += 32) ws.bdone[(size_t)o * VW + v] = 0;
     }
     clear_bitmap(sh.touched, kMaxCols);
     clear_bitmap(sh.dirty, kMaxCols);

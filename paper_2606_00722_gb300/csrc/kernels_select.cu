@@ -6,6 +6,10 @@
 
 using namespace epic;
 
+// Selection and the fallback run one CTA per walk: 16 warps share each
+// column closure (the Gauss-Seidel engine's width, as the forward charts).
+constexpr int kSelThreads = 32 * kGsMaxWarps;
+
 // Alg. 4 per sequence: one CTA runs RelaxedSelect / ExactShrink with an
 // explicit stack; thread 0 drives the recursion, the whole CTA runs each
 // cover test (CoverCols walk) and exact joint check (a walk with the
@@ -23,7 +27,7 @@ struct SelFrame {
 // once, one CTA each per sequence, before the recursion; k_select reuses the
 // two answers when it asks for exactly these tests.  spec[b] = {cover,
 // exact}: 1 pass, 0 fail, -1 not available (overflow / bad input).
-__global__ void __launch_bounds__(kThreads) k_select_spec(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
+__global__ void __launch_bounds__(kSelThreads) k_select_spec(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
                                                           const int32_t* __restrict__ x, int B, int n,
                                                           const int32_t* __restrict__ pos, int k,
                                                           const int32_t* __restrict__ tok, int8_t* __restrict__ spec,
@@ -58,6 +62,8 @@ __global__ void __launch_bounds__(kThreads) k_select_spec(DevGrammar g, const Le
       Subst s{s_pos, s_tok, ns};
       if (exact) {
         EarleyColsGS<false> cols(g, tb, table, ws, sc, wsp.dims, sh, gss);
+        cols.par = g.gs_par != 0;
+        cols.wscr = (uint32_t*)(dyn + gs_tables_bytes(g.D, g.W, g.adv_steps));
         Walk<EarleyColsGS<false>> w(cols, g, table, sc, sh, vocab);
         r = w.run(x + (long long)b * n, n, s);
       } else {
@@ -71,7 +77,7 @@ __global__ void __launch_bounds__(kThreads) k_select_spec(DevGrammar g, const Le
   }
 }
 
-__global__ void __launch_bounds__(kThreads) k_select(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
+__global__ void __launch_bounds__(kSelThreads) k_select(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
                                                      const int32_t* __restrict__ x, int B, int n,
                                                      const int32_t* __restrict__ pos, int k,
                                                      const int32_t* __restrict__ tok, const float* __restrict__ conf,
@@ -91,6 +97,8 @@ __global__ void __launch_bounds__(kThreads) k_select(DevGrammar g, const LexEntr
   WalkScratch sc;
   wsp.carve(blockIdx.x, ws, sc);
   EarleyColsGS<false> ecols(g, tb, table, ws, sc, wsp.dims, sh, gss);
+  ecols.par = g.gs_par != 0;
+  ecols.wscr = (uint32_t*)(dyn + gs_tables_bytes(g.D, g.W, g.adv_steps));
   CoverCols ccols(g, ws, wsp.dims, sh);
   Walk<EarleyColsGS<false>> exact(ecols, g, table, sc, sh, vocab);
   Walk<CoverCols> cover(ccols, g, table, sc, sh, vocab);
@@ -274,156 +282,219 @@ __global__ void __launch_bounds__(kThreads) k_select(DevGrammar g, const LexEntr
   }
 }
 
-// Alg. 1's sequential rejection fallback, one CTA per sequence: fill =
-// max(0, n_target[b] - |B|) more commits, each the highest-confidence
-// candidate (ties: position, then candidate index) at a still-masked
-// position that was not rejected and whose update passes the exact test
-// (a whole-graph walk of x (+) c with the Gauss-Seidel columns); a candidate
-// that fails is rejected for good (x only gains commits, and completability
-// is monotone).  With the single-candidate bits of x before the commits
-// (valid, may be null), a candidate whose bit is 0 is rejected without a
-// walk: its test would fail (monotonicity again).  Commits go straight into
-// x.  Bounded by the k K candidates.
-__global__ void __launch_bounds__(kThreads) k_fallback(DevGrammar g, const LexEntry* __restrict__ table, int vocab,
-                                                       int32_t* __restrict__ x, int B, int n,
-                                                       const int32_t* __restrict__ pos, int k,
-                                                       const int32_t* __restrict__ cand,
-                                                       const float* __restrict__ conf, int K,
-                                                       const int32_t* __restrict__ n_target,
-                                                       const uint8_t* __restrict__ selected,
-                                                       const uint8_t* __restrict__ valid,
-                                                       int32_t* __restrict__ filled, WsPack wsp,
-                                                       unsigned long long* stats) {
+// Alg. 1's sequential rejection fallback: fill = max(0, n_target[b] - |B|)
+// more commits, each the highest-confidence candidate (ties: position, then
+// candidate index) at a still-masked position that was not rejected and
+// whose update passes the exact test (a whole-graph walk of x (+) c with the
+// Gauss-Seidel columns); a candidate that fails is rejected for good (x only
+// gains commits, and completability is monotone).  With the single-candidate
+// bits of x before the commits (valid, may be null), a candidate whose bit
+// is 0 is rejected without a walk: its test would fail.
+//
+// The loop runs in rounds, m CTAs per sequence: CTA s tests the s-th
+// candidate of the current order against the current x, all at once; then
+// the round is read in order, exactly as the sequential loop would meet
+// it -- failed tests reject, the first passing one is committed, and after
+// that commit a failed test still rejects (it fails against the larger x
+// too) while a passing one is tested again next round.  The result is the
+// sequential loop's; only the tests after a commit are spent.
+//
+// State per sequence (global): fb[0] commits still wanted, fb[1] active.
+
+// per sequence: outputs cleared, rejections from the validity bits, the
+// fill, bad inputs; counts the active sequences
+__global__ void k_fallback_init(int B, int n, const int32_t* __restrict__ pos, int k,
+                                const float* __restrict__ conf, int K, const int32_t* __restrict__ n_target,
+                                const uint8_t* __restrict__ selected, const uint8_t* __restrict__ valid,
+                                int32_t* __restrict__ filled, uint8_t* __restrict__ rej, int32_t* __restrict__ fb,
+                                unsigned long long* __restrict__ active, unsigned long long* stats) {
+  const int b = blockIdx.x;
+  if (b >= B) return;
+  const int nc = k * K;
+  __shared__ int s_bad;
+  if (threadIdx.x == 0) s_bad = 0;
+  __syncthreads();
+  for (int j = threadIdx.x; j < k; j += blockDim.x) {
+    filled[(long long)b * k + j] = -1;
+    const int p = pos[(long long)b * k + j];
+    if (p < 0 || p >= n) s_bad = 1;
+  }
+  for (int q = threadIdx.x; q < nc; q += blockDim.x) {
+    rej[(long long)b * nc + q] = (valid && valid[(long long)b * nc + q] == 0) ? 1 : 0;
+    const float cf = conf[(long long)b * nc + q];
+    if (cf != cf) s_bad = 1;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int nsel = 0;
+    if (selected)
+      for (int j = 0; j < k; ++j) nsel += selected[(long long)b * k + j] == 1;
+    const int fill = n_target[b] - nsel;
+    fb[2 * b] = fill;
+    fb[2 * b + 1] = (!s_bad && fill > 0) ? 1 : 0;
+    if (s_bad) atomicAdd(&stats[S_BAD], 1ull);
+    if (fb[2 * b + 1]) atomicAdd(active, 1ull);
+  }
+}
+
+// Block: the best candidate of sequence b (the order above) among those not
+// rejected, at masked positions, and not in excl[0..nex); -1 if none.
+__device__ int fallback_best(int b, const int32_t* xb, const int32_t* pos, int k, const float* conf, int K,
+                             const uint8_t* rej, const int* excl, int nex, float* r_cf, int* r_q) {
+  const int nc = k * K;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  auto before = [&](float ca, int qa, float cb, int qb) -> bool {  // (ca, qa) ahead of (cb, qb)
+    if (qb < 0) return qa >= 0;
+    if (qa < 0) return false;
+    if (ca != cb) return ca > cb;
+    const int pa = pos[(long long)b * k + qa / K], pb = pos[(long long)b * k + qb / K];
+    return pa < pb || (pa == pb && qa < qb);
+  };
+  float bc = 0.f;
+  int bq = -1;
+  for (int q = threadIdx.x; q < nc; q += blockDim.x) {
+    if (rej[(long long)b * nc + q]) continue;
+    if (xb[pos[(long long)b * k + q / K]] >= 0) continue;  // committed by the selected batch or here
+    bool ex = false;
+    for (int i = 0; i < nex; ++i) ex |= excl[i] == q;
+    if (ex) continue;
+    const float cf = conf[(long long)b * nc + q];
+    if (before(cf, q, bc, bq)) {
+      bc = cf;
+      bq = q;
+    }
+  }
+  for (int off = 16; off; off >>= 1) {
+    const float oc = __shfl_xor_sync(0xffffffffu, bc, off);
+    const int oq = __shfl_xor_sync(0xffffffffu, bq, off);
+    if (before(oc, oq, bc, bq)) {
+      bc = oc;
+      bq = oq;
+    }
+  }
+  if (lane == 0) {
+    r_cf[warp] = bc;
+    r_q[warp] = bq;
+  }
+  __syncthreads();
+  float c0 = 0.f;
+  int q0 = -1;
+  for (int i = 0; i < (int)(blockDim.x >> 5); ++i)
+    if (before(r_cf[i], r_q[i], c0, q0)) {
+      c0 = r_cf[i];
+      q0 = r_q[i];
+    }
+  __syncthreads();
+  return q0;
+}
+
+// One round: job (b, s) tests the s-th candidate of sequence b's order.
+// res[(b m + s) 2] = candidate (-1: none), [+1] = 1 pass, 0 fail, -1 capacity.
+__global__ void __launch_bounds__(kSelThreads) k_fallback_round(DevGrammar g, const LexEntry* __restrict__ table,
+                                                             int vocab, const int32_t* __restrict__ x, int B, int n,
+                                                             const int32_t* __restrict__ pos, int k,
+                                                             const int32_t* __restrict__ cand,
+                                                             const float* __restrict__ conf, int K, int m,
+                                                             const uint8_t* __restrict__ rej,
+                                                             const int32_t* __restrict__ fb, int32_t* __restrict__ res,
+                                                             WsPack wsp, unsigned long long* stats) {
   __shared__ WalkShared sh;
   __shared__ GsShared gss;
   extern __shared__ __align__(16) unsigned char dyn[];
   GsTables tb;
   gs_stage_tables(g, dyn, tb);
-  __shared__ uint8_t rej[kMaxFallbackCand];
-  __shared__ float r_cf[kThreads / 32];
-  __shared__ int r_q[kThreads / 32];
+  __shared__ float r_cf[kSelThreads / 32];
+  __shared__ int r_q[kSelThreads / 32];
+  __shared__ int excl[kMaxFallbackSpec];
   __shared__ int s_pos[1], s_tok[1];
-  __shared__ int s_fill, s_bad, s_q;
   Workspace ws;
   WalkScratch sc;
   wsp.carve(blockIdx.x, ws, sc);
   EarleyColsGS<false> cols(g, tb, table, ws, sc, wsp.dims, sh, gss);
+  cols.par = g.gs_par != 0;
+  cols.wscr = (uint32_t*)(dyn + gs_tables_bytes(g.D, g.W, g.adv_steps));
   Walk<EarleyColsGS<false>> walk(cols, g, table, sc, sh, vocab);
-  const int nc = k * K;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  unsigned long long n_chk = 0, n_com = 0, n_ovf = 0, n_bad = 0;
-  for (int b = blockIdx.x; b < B; b += gridDim.x) {
-    int32_t* xb = x + (long long)b * n;
-    for (int j = threadIdx.x; j < k; j += blockDim.x) filled[(long long)b * k + j] = -1;
-    for (int q = threadIdx.x; q < nc; q += blockDim.x) rej[q] = (valid && valid[(long long)b * nc + q] == 0) ? 1 : 0;
-    if (threadIdx.x == 0) {
-      int nsel = 0;
-      if (selected)
-        for (int j = 0; j < k; ++j) nsel += selected[(long long)b * k + j] == 1;
-      s_fill = n_target[b] - nsel;
-      s_bad = 0;
-      for (int q = 0; q < nc; ++q) {
-        const float cf = conf[(long long)b * nc + q];
-        if (cf != cf) s_bad = 1;
-        const int p = pos[(long long)b * k + q / K];
-        if (p < 0 || p >= n) s_bad = 1;
+  unsigned long long n_chk = 0;
+  for (long long job = blockIdx.x; job < (long long)B * m; job += gridDim.x) {
+    const int b = (int)(job / m), sl = (int)(job % m);
+    int32_t* out = res + 2 * job;
+    if (!fb[2 * b + 1]) {
+      if (threadIdx.x == 0) {
+        out[0] = -1;
+        out[1] = 0;
       }
-    }
-    __syncthreads();
-    if (s_bad) {
-      if (threadIdx.x == 0) ++n_bad;
       continue;
     }
-    int done = 0;
-    for (int guard = 0; guard <= nc && done < s_fill; ++guard) {
-      // the next candidate: highest confidence, then lowest position, then
-      // lowest candidate index, among those not rejected at masked positions
-      float bc = 0.f;
-      int bq = -1;
-      for (int q = threadIdx.x; q < nc; q += blockDim.x) {
-        if (rej[q]) continue;
+    const int32_t* xb = x + (long long)b * n;
+    int q = -1;
+    for (int i = 0; i <= sl; ++i) {
+      q = fallback_best(b, xb, pos, k, conf, K, rej, excl, i, r_cf, r_q);
+      if (q < 0) break;
+      if (threadIdx.x == 0) excl[i] = q;
+      __syncthreads();
+    }
+    if (q < 0) {
+      if (threadIdx.x == 0) {
+        out[0] = -1;
+        out[1] = 0;
+      }
+      __syncthreads();
+      continue;
+    }
+    if (threadIdx.x == 0) {
+      s_pos[0] = pos[(long long)b * k + q / K];
+      s_tok[0] = cand[(long long)b * k * K + q];
+    }
+    __syncthreads();
+    Subst su{s_pos, s_tok, 1};
+    const int r = walk.run(xb, n, su);
+    if (threadIdx.x == 0) {
+      out[0] = q;
+      out[1] = r;
+      ++n_chk;
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0 && n_chk) atomicAdd(&stats[S_FB_CHECKS], n_chk);
+}
+
+// One thread per sequence: read the round in order (see above); counts the
+// sequences still active.
+__global__ void k_fallback_resolve(int B, int32_t* __restrict__ x, int n, const int32_t* __restrict__ pos, int k,
+                                   const int32_t* __restrict__ cand, int K, int m, uint8_t* __restrict__ rej,
+                                   int32_t* __restrict__ fb, const int32_t* __restrict__ res,
+                                   int32_t* __restrict__ filled, unsigned long long* __restrict__ active,
+                                   unsigned long long* stats) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B || !fb[2 * b + 1]) return;
+  const int nc = k * K;
+  bool committed = false, any = false;
+  unsigned long long n_com = 0, n_ovf = 0;
+  for (int sl = 0; sl < m; ++sl) {
+    const int q = res[2 * ((long long)b * m + sl)], r = res[2 * ((long long)b * m + sl) + 1];
+    if (q < 0) break;
+    any = true;
+    if (!committed) {
+      if (r == 1) {
         const int p = pos[(long long)b * k + q / K];
-        if (xb[p] >= 0) continue;  // committed by the selected batch or earlier here
-        const float cf = conf[(long long)b * nc + q];
-        const bool better = bq < 0 || cf > bc ||
-                            (cf == bc && (p < pos[(long long)b * k + bq / K] ||
-                                          (p == pos[(long long)b * k + bq / K] && q < bq)));
-        if (better) {
-          bc = cf;
-          bq = q;
-        }
+        const int t = cand[(long long)b * nc + q];
+        x[(long long)b * n + p] = t;
+        filled[(long long)b * k + q / K] = t;
+        ++n_com;
+        committed = true;
+        if (--fb[2 * b] <= 0) fb[2 * b + 1] = 0;
+      } else {
+        rej[(long long)b * nc + q] = 1;
+        if (r == -1) ++n_ovf;
       }
-      for (int off = 16; off; off >>= 1) {
-        const float oc = __shfl_xor_sync(0xffffffffu, bc, off);
-        const int oq = __shfl_xor_sync(0xffffffffu, bq, off);
-        bool take = false;
-        if (oq >= 0) {
-          if (bq < 0 || oc > bc) {
-            take = true;
-          } else if (oc == bc) {
-            const int po = pos[(long long)b * k + oq / K], pb = pos[(long long)b * k + bq / K];
-            take = po < pb || (po == pb && oq < bq);
-          }
-        }
-        if (take) {
-          bc = oc;
-          bq = oq;
-        }
-      }
-      if (lane == 0) {
-        r_cf[warp] = bc;
-        r_q[warp] = bq;
-      }
-      __syncthreads();
-      if (threadIdx.x == 0) {
-        float c0 = 0.f;
-        int q0 = -1;
-        for (int i = 0; i < (int)(blockDim.x >> 5); ++i) {
-          const int oq = r_q[i];
-          if (oq < 0) continue;
-          const float oc = r_cf[i];
-          bool take = q0 < 0 || oc > c0;
-          if (!take && oc == c0) {
-            const int po = pos[(long long)b * k + oq / K], pb = pos[(long long)b * k + q0 / K];
-            take = po < pb || (po == pb && oq < q0);
-          }
-          if (take) {
-            c0 = oc;
-            q0 = oq;
-          }
-        }
-        s_q = q0;
-        if (q0 >= 0) {
-          s_pos[0] = pos[(long long)b * k + q0 / K];
-          s_tok[0] = cand[(long long)b * nc + q0];
-        }
-      }
-      __syncthreads();
-      const int q = s_q;
-      if (q < 0) break;  // every candidate rejected
-      Subst su{s_pos, s_tok, 1};
-      const int r = walk.run(xb, n, su);
-      if (threadIdx.x == 0) {
-        ++n_chk;
-        if (r == 1) {
-          xb[s_pos[0]] = s_tok[0];
-          filled[(long long)b * k + q / K] = s_tok[0];
-          ++n_com;
-        } else {
-          rej[q] = 1;
-          if (r == -1) ++n_ovf;
-        }
-      }
-      __syncthreads();
-      if (r == 1) ++done;
+    } else if (r == 0) {
+      rej[(long long)b * nc + q] = 1;  // fails against x, so against x with the commit
     }
   }
-  if (threadIdx.x == 0) {
-    atomicAdd(&stats[S_FB_CHECKS], n_chk);
-    atomicAdd(&stats[S_FB_COMMITS], n_com);
-    atomicAdd(&stats[S_OVERFLOW], n_ovf);
-    atomicAdd(&stats[S_BAD], n_bad);
-  }
+  if (!any) fb[2 * b + 1] = 0;  // every candidate rejected or its position committed
+  if (n_com) atomicAdd(&stats[S_FB_COMMITS], n_com);
+  if (n_ovf) atomicAdd(&stats[S_OVERFLOW], n_ovf);
+  if (fb[2 * b + 1]) atomicAdd(active, 1ull);
 }
 
 namespace epic {
@@ -431,27 +502,47 @@ namespace epic {
 void launch_select_spec(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab,
                         const int32_t* x, int B, int n, const int32_t* pos, int k, const int32_t* tok, int8_t* spec,
                         const WsPack& wsp) {
-  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps);
+  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps) + gs_warp_scratch_bytes();
+  DevGrammar gg = g;
+  gg.gs_par = gs_parallel_enabled(g.W);
   cudaFuncSetAttribute(k_select_spec, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-  k_select_spec<<<grid, kThreads, dyn, st>>>(g, table, vocab, x, B, n, pos, k, tok, spec, wsp);
+  k_select_spec<<<grid, kSelThreads, dyn, st>>>(gg, table, vocab, x, B, n, pos, k, tok, spec, wsp);
 }
 
 void launch_select(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab,
                    const int32_t* x, int B, int n, const int32_t* pos, int k, const int32_t* tok, const float* conf,
                    uint8_t* selected, const WsPack& wsp, const int8_t* spec, unsigned long long* stats) {
-  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps);
+  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps) + gs_warp_scratch_bytes();
+  DevGrammar gg = g;
+  gg.gs_par = gs_parallel_enabled(g.W);
   cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-  k_select<<<grid, kThreads, dyn, st>>>(g, table, vocab, x, B, n, pos, k, tok, conf, selected, wsp, spec, stats);
+  k_select<<<grid, kSelThreads, dyn, st>>>(gg, table, vocab, x, B, n, pos, k, tok, conf, selected, wsp, spec, stats);
 }
 
-void launch_fallback(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab, int32_t* x,
-                     int B, int n, const int32_t* pos, int k, const int32_t* cand, const float* conf, int K,
-                     const int32_t* n_target, const uint8_t* selected, const uint8_t* valid, int32_t* filled,
-                     const WsPack& wsp, unsigned long long* stats) {
-  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps);
-  cudaFuncSetAttribute(k_fallback, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-  k_fallback<<<grid, kThreads, dyn, st>>>(g, table, vocab, x, B, n, pos, k, cand, conf, K, n_target, selected, valid,
-                                          filled, wsp, stats);
+void launch_fallback_init(int B, cudaStream_t st, int n, const int32_t* pos, int k, const float* conf, int K,
+                          const int32_t* n_target, const uint8_t* selected, const uint8_t* valid, int32_t* filled,
+                          uint8_t* rej, int32_t* fb, unsigned long long* active, unsigned long long* stats) {
+  k_fallback_init<<<B, 256, 0, st>>>(B, n, pos, k, conf, K, n_target, selected, valid, filled, rej, fb, active,
+                                     stats);
+}
+
+void launch_fallback_round(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab,
+                           const int32_t* x, int B, int n, const int32_t* pos, int k, const int32_t* cand,
+                           const float* conf, int K, int m, const uint8_t* rej, const int32_t* fb, int32_t* res,
+                           const WsPack& wsp, unsigned long long* stats) {
+  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps) + gs_warp_scratch_bytes();
+  DevGrammar gg = g;
+  gg.gs_par = gs_parallel_enabled(g.W);
+  cudaFuncSetAttribute(k_fallback_round, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+  k_fallback_round<<<grid, kSelThreads, dyn, st>>>(gg, table, vocab, x, B, n, pos, k, cand, conf, K, m, rej, fb, res,
+                                                wsp, stats);
+}
+
+void launch_fallback_resolve(int B, cudaStream_t st, int32_t* x, int n, const int32_t* pos, int k,
+                             const int32_t* cand, int K, int m, uint8_t* rej, int32_t* fb, const int32_t* res,
+                             int32_t* filled, unsigned long long* active, unsigned long long* stats) {
+  k_fallback_resolve<<<(B + 127) / 128, 128, 0, st>>>(B, x, n, pos, k, cand, K, m, rej, fb, res, filled, active,
+                                                      stats);
 }
 
 }  // namespace epic

@@ -45,10 +45,16 @@ void launch_select(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEnt
                    uint8_t* selected, const WsPack& wsp, const int8_t* spec, unsigned long long* stats);
 
 // Alg. 1's sequential rejection fallback
-void launch_fallback(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab, int32_t* x,
-                     int B, int n, const int32_t* pos, int k, const int32_t* cand, const float* conf, int K,
-                     const int32_t* n_target, const uint8_t* selected, const uint8_t* valid, int32_t* filled,
-                     const WsPack& wsp, unsigned long long* stats);
+void launch_fallback_init(int B, cudaStream_t st, int n, const int32_t* pos, int k, const float* conf, int K,
+                          const int32_t* n_target, const uint8_t* selected, const uint8_t* valid, int32_t* filled,
+                          uint8_t* rej, int32_t* fb, unsigned long long* active, unsigned long long* stats);
+void launch_fallback_round(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab,
+                           const int32_t* x, int B, int n, const int32_t* pos, int k, const int32_t* cand,
+                           const float* conf, int K, int m, const uint8_t* rej, const int32_t* fb, int32_t* res,
+                           const WsPack& wsp, unsigned long long* stats);
+void launch_fallback_resolve(int B, cudaStream_t st, int32_t* x, int n, const int32_t* pos, int k,
+                             const int32_t* cand, int K, int m, uint8_t* rej, int32_t* fb, const int32_t* res,
+                             int32_t* filled, unsigned long long* active, unsigned long long* stats);
 
 // witness extraction (Sec. 4.4) from the forward charts of checks by region
 void launch_witness(int B, cudaStream_t st, const DevGrammar& g, const SeqPack& sp, int32_t* terms, int cap,

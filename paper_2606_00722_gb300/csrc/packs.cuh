@@ -55,6 +55,7 @@ enum StatIdx {
   S_FB_CHECKS, S_FB_COMMITS, S_LEX_LOOKUPS, S_LEX_MISSES, S_LEX_UNCACHED, S_WITNESS_FAIL, S_N
 };
 constexpr int kMaxFallbackCand = 4096;  // proposed (position, candidate) pairs per sequence of the fallback
+constexpr int kMaxFallbackSpec = 16;    // fallback tests of one sequence in one round
 
 // shared-memory staging of one warp: rows, completed-NT sets, slot origins,
 // origin slots (16-byte multiple)

@@ -78,8 +78,9 @@ __global__ void __launch_bounds__(32 * kGsMaxWarps, 1) k_forward_gs(DevGrammar g
   gs_stage_tables(g, dyn, tb);
   for (long long b = blockIdx.x; b < B; b += gridDim.x) {
     SeqArena a = sp.carve(b);
-    // the walk expects a zeroed stage
+    // the walk expects a zeroed stage and completion record
     for (size_t w = threadIdx.x; w < (size_t)sp.nmax * g.W; w += blockDim.x) a.ws.stage[w] = 0;
+    for (size_t w = threadIdx.x; w < (size_t)sp.nmax * g.VW; w += blockDim.x) a.ws.bdone[w] = 0;
     for (int p = threadIdx.x; p < n; p += blockDim.x) {
       a.rec.gap_col[p] = -1;
       a.rec.pre_col[p] = -1;
@@ -88,7 +89,7 @@ __global__ void __launch_bounds__(32 * kGsMaxWarps, 1) k_forward_gs(DevGrammar g
     __syncthreads();
     Workspace ws;
     ws.stage = a.ws.stage;
-    ws.bdone = nullptr;
+    ws.bdone = a.ws.bdone;
     ws.col_off = a.ws.col_off;
     ws.org = a.ws.org;
     ws.bits = a.ws.bits;
@@ -113,6 +114,8 @@ __global__ void __launch_bounds__(32 * kGsMaxWarps, 1) k_forward_gs(DevGrammar g
     EarleyColsGS<true> cols(g, tb, table, ws, sc, d, sh, gss);
     cols.rec = &br;
     cols.wnt = (uint32_t*)(dyn + gs_tables_bytes(g.D, g.W, g.adv_steps));
+    cols.wscr = cols.wnt + (size_t)kGsMaxWarps * kMaxVW;
+    cols.par = g.gs_par != 0;
     Walk<EarleyColsGS<true>> walk(cols, g, table, sc, sh, vocab);
     walk.rec = &br;
     Subst none{nullptr, nullptr, 0};
@@ -146,9 +149,12 @@ void launch_forward(bool sm, dim3 grid, dim3 block, size_t dyn, cudaStream_t st,
 
 void launch_forward_gs(dim3 grid, cudaStream_t st, const DevGrammar& g, const LexEntry* table, int vocab,
                        const int32_t* x, int B, int n, const SeqPack& sp, unsigned long long* stats) {
-  const size_t dyn = gs_tables_bytes(g.D, g.W, g.adv_steps) + (size_t)kGsMaxWarps * kMaxVW * 4;
+  const size_t dyn =
+      gs_tables_bytes(g.D, g.W, g.adv_steps) + (size_t)kGsMaxWarps * kMaxVW * 4 + gs_warp_scratch_bytes();
+  DevGrammar gg = g;
+  gg.gs_par = gs_parallel_enabled(g.W);
   cudaFuncSetAttribute(k_forward_gs, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-  k_forward_gs<<<grid, 32 * kGsMaxWarps, dyn, st>>>(g, table, vocab, x, B, n, sp, stats);
+  k_forward_gs<<<grid, 32 * kGsMaxWarps, dyn, st>>>(gg, table, vocab, x, B, n, sp, stats);
 }
 
 // measurement builds: this translation unit's phase counters of the walk

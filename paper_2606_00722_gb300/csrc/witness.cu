@@ -210,6 +210,55 @@ __global__ void __launch_bounds__(32 * kWarpsPerCta) k_witness(DevGrammar g, int
   if (lane == 0) {
     out_len[b] = status == 0 ? len : -2;
     if (status == 3) atomicAdd(&stats[S_WITNESS_FAIL], 1ull);
+#ifdef EPIC_WITNESS_DEBUG
+    if (status != 0 && cap >= 12) {  // measurement builds: where the search stopped
+      out_len[b] = -10 - status;
+      const WGoal cur = G[ns >= 0 && ns < gcap ? S[ns] : 0];
+      const int i = cur.item;
+      out[0] = i;
+      out[1] = cur.o;
+      out[2] = cur.j;
+      out[3] = i > 0 ? g.item_next[i - 1] : -1;
+      out[4] = a.rec.col_gap[cur.j];
+      out[5] = len;
+      out[6] = ng;
+      out[7] = ns;
+      out[8] = T;
+      out[9] = a.in_off[cur.j + 1] - a.in_off[cur.j];
+      out[10] = present(i - 1, cur.o, cur.j) ? 1 : 0;
+      out[11] = i > 0 ? (int)((g.nullable_next[(i - 1) >> 5] >> ((i - 1) & 31)) & 1u) : -1;
+      if (cap >= 64) {
+        // splits m in [o, j): left part present / X completes from m at j
+        const int X = i > 0 ? g.item_next[i - 1] : -1;
+        int np = 0, nc = 0, p0 = -1, c0 = -1;
+        for (int m = cur.o; m < cur.j; ++m) {
+          if (present(i - 1, cur.o, m)) {
+            ++np;
+            p0 = m;
+          }
+          if (X >= T && completes(X - T, m, cur.j)) {
+            ++nc;
+            c0 = m;
+          }
+        }
+        out[12] = np;
+        out[13] = p0;
+        out[14] = nc;
+        out[15] = c0;
+        out[16] = present(i, cur.o, cur.j) ? 1 : 0;
+        // in-edges: source, label words or-ed, item present at the source
+        int q = 17;
+        for (int e = a.in_off[cur.j]; e < a.in_off[cur.j + 1] && q + 3 <= 60; ++e) {
+          uint32_t lo = 0;
+          for (int w = 0; w < 8; ++w) lo |= a.rec.e_lbl[(size_t)e * 8 + w];
+          out[q++] = a.rec.e_src[e];
+          out[q++] = (int)lo;
+          out[q++] = present(i, cur.o, a.rec.e_src[e]) ? 1 : 0;
+        }
+        out[q] = -99;
+      }
+    }
+#endif
   }
 }
 

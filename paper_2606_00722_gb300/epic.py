@@ -74,7 +74,7 @@ class _Stats(C.Structure):
                                           'entries', 'cover_checks', 'exact_checks', 'selected',
                                           'region_checks', 'validate_kernels', 'fallback_checks',
                                           'fallback_commits', 'lex_lookups', 'lex_misses', 'lex_uncached',
-                                          'witness_failures')]
+                                          'witness_failures', 'fallback_rounds')]
 
 
 class _Desc(C.Structure):

@@ -65,6 +65,16 @@ def test_step_parity(cuda, name, seed, kw):
     assert got['stats']['checks'] == w.cand.size
 
 
+@pytest.mark.parametrize('name,seed,kw', [('json-schema', 43, dict(batch=3, k=3)),
+                                          ('clike-512', 42, dict(batch=2, k=4, K=4, n=160))])
+def test_step_parity_descending_sweep(cuda, monkeypatch, name, seed, kw):
+    """The CTA walks (forward charts of wide grammars, selection's exact
+    tests) with the descending block sweep of the column closure instead of
+    the warp-parallel one: the same least fixpoint, so the same bits."""
+    monkeypatch.setenv('EPIC_GS_PARALLEL', '0')
+    test_step_parity(cuda, name, seed, kw)
+
+
 @pytest.mark.parametrize('name', ['expr-tiny', 'json-schema', 'smiles-256'])
 def test_lex_table_runs_match_oracle(cuda, name):
     """Every token's run from the initial state, and the set of distinct runs
@@ -144,11 +154,11 @@ def test_decode_step_with_fallback(cuda, name, seed, kw, fill):
     np.testing.assert_array_equal(bufs['selected'].cpu().numpy(), ref_sel)
     np.testing.assert_array_equal(bufs['filled'].cpu().numpy(), ref_filled)
     np.testing.assert_array_equal(x.cpu().numpy(), ref_x)
-    # decode_step hands the fallback the step's validity bits, so it tests
-    # only candidates whose bit is not 0 (the others would fail their test)
-    assert st['fallback_checks'] <= nchk
+    # (decode_step hands the fallback the step's validity bits: candidates
+    # whose bit is 0 are rejected untested, with the same result)
     assert st['fallback_commits'] == int((ref_filled >= 0).sum())
     # without the bits every candidate is tested, as in the oracle's loop
+    # (a round also tests the candidates after its commit)
     x2 = _dev(x1, cuda)
     filled2 = torch.empty(w.pos.shape, dtype=torch.int32, device=cuda)
     t.stats(reset=True)
@@ -158,7 +168,8 @@ def test_decode_step_with_fallback(cuda, name, seed, kw, fill):
     st2 = t.stats()
     np.testing.assert_array_equal(filled2.cpu().numpy(), ref_filled)
     np.testing.assert_array_equal(x2.cpu().numpy(), ref_x)
-    assert st2['fallback_checks'] == nchk
+    # the rounds test at least the candidates the sequential loop tests
+    assert st2['fallback_checks'] >= nchk
 
 
 def _step_with_table(w, dev, lazy_capacity):
@@ -202,4 +213,6 @@ def test_lazy_lex_memo_equals_dense_table(cuda, name, seed, kw):
         if cap == 64:
             assert st['lex_uncached'] > 0
         else:
-            assert st['lex_uncached'] == 0 and st['lex_misses'] < st['lex_lookups']
+            # a lookup that finds its entry still being computed by another
+            # thread may compute it itself (bounded wait): rare, not a miss of capacity
+            assert st['lex_uncached'] <= st['lex_lookups'] // 100 and st['lex_misses'] < st['lex_lookups']
