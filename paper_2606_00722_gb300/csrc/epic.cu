@@ -1070,7 +1070,7 @@ epic_status epic_extract_witness(const epic_grammar* g, const epic_lexer_table* 
   SeqPack sp;
   epic_status s = region_prepare(g, t, d_x, B, n, sp, st);
   if (s != EPIC_OK) return s;
-  const size_t per = witness_goal_bytes(cap);
+  const size_t per = witness_scratch_bytes(cap, t->dgl.D, t->dgl.W, t->dgl.VW);
   s = grow(t, &t->d_wit, &t->wit_bytes, per * (size_t)B);
   if (s != EPIC_OK) return s;
   launch_witness(B, st, t->dgl, sp, d_terms, cap, d_len, t->d_wit, t->d_stats);

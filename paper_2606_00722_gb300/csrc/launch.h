@@ -59,7 +59,7 @@ void launch_fallback_resolve(int B, cudaStream_t st, int32_t* x, int n, const in
 // witness extraction (Sec. 4.4) from the forward charts of checks by region
 void launch_witness(int B, cudaStream_t st, const DevGrammar& g, const SeqPack& sp, int32_t* terms, int cap,
                     int32_t* out_len, void* scratch, unsigned long long* stats);
-size_t witness_goal_bytes(int cap);  // goal and stack scratch per sequence
+size_t witness_scratch_bytes(int cap, int D, int W, int VW);  // scratch per sequence
 
 // measurement builds (EPIC_PHASE_TIMERS): the walk's phase counters of one
 // translation unit, added into out16 (reset: zeroed afterwards)
