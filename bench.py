@@ -42,6 +42,9 @@ def parse():
     ap.add_argument('--gpus', type=int, default=1)
     ap.add_argument('--steps', type=int, default=5)
     ap.add_argument('--warmup', type=int, default=3)
+    # clike-512 (32 x 512, k 8, K 32) is the largest workload whose steps fit
+    # a bench run of minutes; random-stress-1024 (64 x 1024, k 16, K 32) runs
+    # with --workload random-stress-1024 at several minutes per step
     ap.add_argument('--workload', default='clike-512')
     ap.add_argument('--impl', default='epic', choices=['epic', 'reference'])
     ap.add_argument('--seed', type=int, default=42)
@@ -479,6 +482,7 @@ def main():
             'config': {'workload': args.workload, 'batch': w.B, 'seq_len': w.n, 'k': w.k, 'K': w.K,
                        'vocab': len(w.vocab), 'l2': 'flushed: 256 MiB write before every step',
                        'parallelism': 'replicas' if world > 1 else 'single'},
+            'step': 'validate, pick, select (Alg. 4), commit, rejection fallback (Alg. 1) with n_t = k',
             'step_latency_us': ms * 1e3, 'validate_checks_per_s': total_checks / (vms / 1e3),
             'valid_fraction': st['valid'] / max(1, st['checks']), 'overflow': st['overflow'],
             'gpu_launches': int(launches), 'validate_path': 'region' if region else 'walk',
