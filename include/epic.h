@@ -78,7 +78,7 @@ typedef struct {
 } epic_grammar_desc;
 
 /*
- * Compile a grammar (Alg. 1 line 1-2: compile the lexical map; the regular
+ * Compile a grammar (Alg. 1, its set-up: compile the lexical map; the regular
  * cover of Sec. 4.3 / App. A.2 is derived from the same tables).  Builds the
  * union lexer DFA (minimized), trims unproductive and unreachable symbols,
  * numbers the dotted items and uploads the device tables to the current
@@ -89,7 +89,7 @@ typedef struct {
 epic_status epic_grammar_create(const epic_grammar_desc* desc, epic_grammar** out);
 void epic_grammar_destroy(epic_grammar* g);
 
-/* Number of lexer DFA states (the "live lexer states" a span after a gap may
+/* Number of lexer DFA states (the states a span after a gap may
  * start in, Sec. 2 / Alg. 2), or -1 for NULL. */
 int32_t epic_grammar_lexer_states(const epic_grammar* g);
 
@@ -139,7 +139,7 @@ epic_status epic_lexer_table_copy(const epic_lexer_table* t, int32_t first_token
                                   void* host_out, size_t out_bytes);
 
 /*
- * Batched validity checks (Sec. 3; Alg. 3 per check; Alg. 1 line 15):
+ * Batched validity checks (Sec. 3; Alg. 3 per check; Alg. 1's validity test):
  *   d_valid[b][j][c] = Valid_G(x_b, {(d_pos[b][j], d_cand[b][j][c])})
  *                    = 1[ L(G) cap C_{x_b (+) (pos, tok)} != empty ].
  * d_x [B][n] int32 (-1 = MASK); d_pos [B][k] int32, each a masked position of
@@ -206,7 +206,7 @@ epic_status epic_validate_batch_noalloc(const epic_grammar* g, const epic_lexer_
                                         int32_t K, uint8_t* d_valid, void* cuda_stream);
 
 /*
- * Candidate set C of Alg. 1 line 7 ("high-confidence candidates"), read as:
+ * Candidate set C of Alg. 1 (each position's best valid candidate), read as:
  * per proposed position, the highest-confidence candidate whose valid bit is
  * 1 (ties: lowest candidate index), else none.  d_cand [B][k][K] int32,
  * d_cand_conf [B][k][K] float32, d_valid [B][k][K] uint8; outputs d_tok [B][k]
@@ -235,15 +235,15 @@ epic_status epic_select_compatible_subset(const epic_grammar* g, const epic_lexe
                                           void* cuda_stream);
 
 /*
- * Commit (Alg. 1 line 10): d_x[b][d_pos[b][j]] = d_tok[b][j] where
+ * Commit (Alg. 1): d_x[b][d_pos[b][j]] = d_tok[b][j] where
  * d_selected[b][j] == 1.  Asynchronous.
  */
 epic_status epic_commit(int32_t* d_x, int32_t B, int32_t n, const int32_t* d_pos, int32_t k,
                         const int32_t* d_tok, const uint8_t* d_selected, void* cuda_stream);
 
 /*
- * Sequential rejection fallback (Alg. 1, the loop that follows the commit of
- * the selected batch B, "if verification fails or commits remain"): for each
+ * Sequential rejection fallback (Alg. 1, the loop after the selected batch B
+ * is committed, run when B fails its test or more commits are wanted): for each
  * of the max(0, d_n_target[b] - |B_b|) commits still wanted, take the
  * highest-confidence candidate over every proposed position and its K
  * candidates whose position is still masked in d_x and that was not
@@ -305,8 +305,8 @@ typedef struct {
   uint64_t bad_inputs;       /* unmasked positions / bad token ids / NaNs      */
   uint64_t columns;          /* Earley chart columns (graph nodes) processed   */
   uint64_t entries;          /* (node, origin) chart entries stored            */
-  uint64_t cover_checks;     /* regular-cover group tests (Alg. 4 line 9)      */
-  uint64_t exact_checks;     /* joint exact checks (Alg. 4 line 21)            */
+  uint64_t cover_checks;     /* regular-cover group tests (Alg. 4, Relaxed)  */
+  uint64_t exact_checks;     /* joint exact checks (Alg. 4, ExactShrink)     */
   uint64_t selected;         /* candidates committed by selection              */
   uint64_t region_checks;    /* of the checks, those answered by region walks
                                 over a per-sequence forward chart            */

@@ -482,8 +482,8 @@ bool earley_valid(const Grammar& g, const Graph& G, bool early_exit, EarleyStats
 }
 
 // ------------------------------------------------------------------ cover
-// Regular cover F_G (Sec. 4.3, App. A.2, App. D.3): the CFG as a recursive
-// transition network, flattened.  States entry(A), exit(A) and (p, j) for
+// Regular cover F_G (Sec. 4.3, App. A.2, App. D.3): one network of states per
+// grammar with its calls flattened.  States entry(A), exit(A) and (p, j) for
 // every production p and dot j.  Every call site, recursive or not, goes to
 // the one shared entry(B); exit(B) returns to every continuation of B.
 struct Cover {
@@ -647,7 +647,7 @@ std::vector<std::pair<int, int>> as_updates(const CandList& c) {
   return u;
 }
 
-// "high-confidence halves": the first ceil(|C|/2) of the confidence order
+// the more confident half: the first ceil(|C|/2) of the confidence order
 void split_halves(const CandList& c, CandList& L, CandList& R) {
   size_t h = (c.size() + 1) / 2;
   L.assign(c.begin(), c.begin() + h);

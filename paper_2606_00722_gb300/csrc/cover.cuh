@@ -1,4 +1,4 @@
-// Regular-cover group test (Sec. 4.3, Alg. 4 line 9): L(F_G) cap L(A_x) != empty
+// Regular-cover group test (Sec. 4.3, Alg. 4's RelaxedSelect): L(F_G) cap L(A_x) != empty
 // by forward state-set simulation of the flattened recursive transition
 // network F_G over the partial-output graph.
 //
