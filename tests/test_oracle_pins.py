@@ -533,6 +533,38 @@ def test_commit_writes_selected_tokens():
 
 
 # ------------------------------------------------------------------ candidate set C
+def load_select_cases():
+    """tests/golden/select_cases.txt as (grammar, n, positions, tokens,
+    confidences, expected selected) rows."""
+    rows = []
+    with open(os.path.join(HERE, 'golden', 'select_cases.txt')) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith('#'):
+                continue
+            gname, n, p, t, c, e = (s.strip() for s in line.split('|'))
+            rows.append((gname, int(n), [int(a) for a in p.split()], [int(a) for a in t.split()],
+                         [float(a) for a in c.split()], [int(a) for a in e.split()]))
+    return rows
+
+
+def test_select_golden():
+    """Alg. 4 (RelaxedSelect, then ExactShrink) on hand-derived cases: sizes
+    one and two, a first half kept while the second fails, ties in confidence
+    ordered by position, and a cover that over-accepts so that ExactShrink
+    must shrink the relaxed set (and, in one case, down to nothing)."""
+    grammars = {'nonrec': (tiny_nonrec(), [b'a', b'b', b'c', b'd', b'e']),
+                'paren': (tiny_paren(), [b'(', b')', b'a', b'b'])}
+    rows = load_select_cases()
+    assert len(rows) >= 9
+    for gname, n, pos, tok, conf, expect in rows:
+        spec, vocab = grammars[gname]
+        O = oracle.Oracle(spec, vocab)
+        x = np.full((1, n), -1, np.int32)
+        sel = O.select(x, np.array([pos], np.int32), np.array([tok], np.int32), np.array([conf], np.float32))
+        assert sel[0].tolist() == expect, (gname, pos, tok, conf, sel[0].tolist())
+
+
 def load_pick_cases():
     """tests/golden/pick_cases.txt as (valid [R][4], conf [R][4], cand [R][4],
     expected token [R], expected confidence [R]); token of line r, index c is
