@@ -535,16 +535,16 @@ def test_commit_writes_selected_tokens():
 # ------------------------------------------------------------------ candidate set C
 def load_select_cases():
     """tests/golden/select_cases.txt as (grammar, n, positions, tokens,
-    confidences, expected selected) rows."""
+    confidences, expected selected, (cover tests, exact tests)) rows."""
     rows = []
     with open(os.path.join(HERE, 'golden', 'select_cases.txt')) as f:
         for line in f:
             line = line.strip()
             if not line or line.startswith('#'):
                 continue
-            gname, n, p, t, c, e = (s.strip() for s in line.split('|'))
+            gname, n, p, t, c, e, k = (s.strip() for s in line.split('|'))
             rows.append((gname, int(n), [int(a) for a in p.split()], [int(a) for a in t.split()],
-                         [float(a) for a in c.split()], [int(a) for a in e.split()]))
+                         [float(a) for a in c.split()], [int(a) for a in e.split()], tuple(int(a) for a in k.split())))
     return rows
 
 
@@ -556,13 +556,14 @@ def test_select_golden():
     grammars = {'nonrec': (tiny_nonrec(), [b'a', b'b', b'c', b'd', b'e']),
                 'paren': (tiny_paren(), [b'(', b')', b'a', b'b'])}
     rows = load_select_cases()
-    assert len(rows) >= 9
-    for gname, n, pos, tok, conf, expect in rows:
+    assert len(rows) >= 10
+    for gname, n, pos, tok, conf, expect, tests in rows:
         spec, vocab = grammars[gname]
         O = oracle.Oracle(spec, vocab)
         x = np.full((1, n), -1, np.int32)
         sel = O.select(x, np.array([pos], np.int32), np.array([tok], np.int32), np.array([conf], np.float32))
         assert sel[0].tolist() == expect, (gname, pos, tok, conf, sel[0].tolist())
+        assert O.last_select_counts == tests, (gname, pos, tok, conf, O.last_select_counts)
 
 
 def load_pick_cases():
