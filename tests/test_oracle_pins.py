@@ -566,6 +566,33 @@ def test_select_golden():
         assert O.last_select_counts == tests, (gname, pos, tok, conf, O.last_select_counts)
 
 
+def test_fallback_golden():
+    """Alg. 1's rejection fallback on hand-derived cases (tests/golden/
+    fallback_cases.txt): commits in confidence order, rejections, positions
+    committed by the selected batch skipped, ties by position then candidate
+    index, n_t no larger than |B|; with the number of exact tests."""
+    O = oracle.Oracle(tiny_nonrec(), [b'a', b'b', b'c', b'd', b'e'])
+    cases = 0
+    with open(os.path.join(HERE, 'golden', 'fallback_cases.txt')) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith('#'):
+                continue
+            xs, ps, ss, cs, fs, nt, ex, ef, et = (v.strip() for v in line.split('|'))
+            x = np.array([[int(v) for v in xs.split()]], np.int32)
+            pos = np.array([[int(v) for v in ps.split()]], np.int32)
+            k = pos.shape[1]
+            sel = np.array([[int(v) for v in ss.split()]], np.uint8)
+            cand = np.array([int(v) for v in cs.split()], np.int32).reshape(1, k, -1)
+            conf = np.array([float(v) for v in fs.split()], np.float32).reshape(1, k, -1)
+            got_x, filled, nchk = O.fallback(x, pos, cand, conf, np.array([int(nt)], np.int32), sel)
+            assert got_x[0].tolist() == [int(v) for v in ex.split()], line
+            assert filled[0].tolist() == [int(v) for v in ef.split()], line
+            assert nchk == int(et), (line, nchk)
+            cases += 1
+    assert cases >= 6
+
+
 def load_pick_cases():
     """tests/golden/pick_cases.txt as (valid [R][4], conf [R][4], cand [R][4],
     expected token [R], expected confidence [R]); token of line r, index c is
