@@ -8,7 +8,7 @@ subset selection with exact shrink, and Alg. 1's sequential rejection
 fallback.  It shares no code with the CUDA path.
 
 Only ``tests/``, ``__graft_entry__.smoke()`` and the benchmark's CPU-baseline
-leg may import this module.
+leg and reference arm may import this module.
 """
 from __future__ import annotations
 

@@ -10,13 +10,15 @@
 //   * the Earley-style graph parser deciding it                     (Alg. 3, App. C.3)
 //   * the flattened recursive-transition-network regular cover      (Sec. 4.3, App. A.2, App. D.3)
 //   * relaxed compatible subset selection + exact shrink            (Alg. 4)
+//   * the sequential rejection fallback                             (Alg. 1)
+//   * membership of a terminal string in a partial output's graph   (witness checks, Sec. 4.4)
 //
 // Where the paper is silent (lexer rule, gap model, cover flattening,
 // tie-breaks) a reading is taken; each is stated where it is implemented
 // below.
 //
-// Only tests, the smoke check and the benchmark's CPU-baseline leg may load
-// this library.  It shares no code, header or table with the CUDA path: it
+// Only tests, the smoke check and the benchmark's CPU-baseline leg and
+// reference arm may load this library.  It shares no code, header or table with the CUDA path: it
 // has its own regex parser, its own lexer (per-terminal Thompson NFAs run by
 // subset simulation, no DFA tables), its own graph and its own parser.
 #include <algorithm>
