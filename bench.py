@@ -483,6 +483,9 @@ def main():
                        'vocab': len(w.vocab), 'l2': 'flushed: 256 MiB write before every step',
                        'parallelism': 'replicas' if world > 1 else 'single'},
             'step': 'validate, pick, select (Alg. 4), commit, rejection fallback (Alg. 1) with n_t = k',
+            'workload_note': ('clike-512 is the default: the largest configuration whose bench run fits minutes '
+                              '(random-stress-1024 took 125 s per step at 8 of its 64 rows)')
+            if args.workload == 'clike-512' else None,
             'step_latency_us': ms * 1e3, 'validate_checks_per_s': total_checks / (vms / 1e3),
             'valid_fraction': st['valid'] / max(1, st['checks']), 'overflow': st['overflow'],
             'gpu_launches': int(launches), 'validate_path': 'region' if region else 'walk',
